@@ -1,0 +1,176 @@
+/*
+ * mixattn — one mixed prefill/decode scheduler iteration on a GB300 (sm_103a).
+ *
+ * The operation is the one the paper's controller observes (§2.1, Eq. 1):
+ * in iteration t, the |D_t| requests that are decoding each bring one new
+ * query token, and one prompt receives a prefill chunk of p_t tokens.  All of
+ * them run causal GQA softmax attention over a paged bf16 KV cache (§2.1,
+ * PagedAttention and chunked prefill; §3.2: attention backend, BF16 precision
+ * and KV layout unchanged), and every new token's K/V is appended to its page
+ * slot.  The iteration call returns the iteration's device-completion time
+ * from CUDA events — the completion-timed signal §6.4 and §9 call for in
+ * place of the scheduler-call interval of §3.2.
+ *
+ * Conventions for every entry point
+ *  - Return value: MX_OK (0) or a negative MX_E* code.  Nothing aborts or
+ *    traps.  A short text for the last failure of a context is available from
+ *    mx_error_detail().
+ *  - bf16 tensors are passed as `void *` to 16-bit elements (bf16 bit
+ *    patterns); int32 arrays as int32_t *.  "device" pointers must be device
+ *    memory of the context's GPU, 16-byte aligned; "host" pointers are read
+ *    before the call returns (they may be reused immediately).
+ *  - All tensors are owned by the caller.  The context owns only a fixed
+ *    workspace allocated by mx_create (work list, split partials, counters,
+ *    error word); no call allocates device memory afterwards.
+ *  - Enqueueing calls are asynchronous on `stream` (a cudaStream_t, NULL for
+ *    the legacy default stream).  One context must not have work in flight on
+ *    two streams at once: its workspace is shared by its calls.
+ *  - Errors a kernel detects (a page id outside the pool, a slot outside the
+ *    pool, an internal wait that timed out) set the context's device error
+ *    word; it is read and cleared by mx_iteration() and mx_sync_status().
+ *
+ * Fixed geometry: head_dim 128, page_size 16, num_q_heads a multiple of
+ * num_kv_heads with num_q_heads / num_kv_heads in {1, 2, 4, 8}.
+ *
+ * Layouts (row-major, bf16):
+ *   q, out   [n_tokens][num_q_heads][128]
+ *   k, v     [n_tokens][num_kv_heads][128]
+ *   k_pool, v_pool  [num_pages][num_kv_heads][16][128]
+ *   page_table      int32 [num_seqs][max_pages_per_seq]; entry = physical page
+ *   slots           int32 [n_tokens]; slot = page * 16 + offset, < 0: skip
+ * Token order in q/k/v/out/slots: the n_decodes decode tokens first (in
+ * decode_seq_ids order), then the p_t chunk tokens in position order.
+ */
+#ifndef MIXATTN_H
+#define MIXATTN_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MX_OK 0
+#define MX_EINVAL (-1)      /* bad argument: null pointer, size, geometry   */
+#define MX_ERANGE_PAGE (-2) /* a page id outside [0, num_pages)             */
+#define MX_ERANGE_SLOT (-3) /* a slot outside [0, num_pages * 16)           */
+#define MX_ECUDA (-4)       /* a CUDA runtime/driver call failed            */
+#define MX_ETIMEOUT (-5)    /* a bounded in-kernel wait gave up             */
+#define MX_EDEVICE (-6)     /* no usable sm_100-family device               */
+#define MX_ECAPACITY (-7)   /* request exceeds the context's geometry       */
+
+/* Device error-word bits (reported through the codes above). */
+#define MX_ERRBIT_PAGE 1u
+#define MX_ERRBIT_SLOT 2u
+#define MX_ERRBIT_TIMEOUT 4u
+
+typedef struct mx_ctx mx_ctx;
+
+/* Geometry and capacity of a context.  num_pages is the page count of every
+ * pool the context will see; max_tokens bounds n_decodes + p_t per call;
+ * max_decodes bounds n_decodes; num_seqs and max_pages_per_seq give the
+ * page-table shape. */
+typedef struct {
+    int32_t num_q_heads;       /* Hq: 16, 32 or 64 in the Qwen3 geometries */
+    int32_t num_kv_heads;      /* Hkv: 8                                  */
+    int32_t head_dim;          /* must be 128                             */
+    int32_t page_size;         /* must be 16                              */
+    int32_t num_pages;         /* pages per pool                          */
+    int32_t num_seqs;          /* page-table rows                         */
+    int32_t max_pages_per_seq; /* page-table row length                   */
+    int32_t max_tokens;        /* max n_decodes + p_t per call            */
+    int32_t max_decodes;       /* max n_decodes per call                  */
+} mx_geom;
+
+/* What one iteration schedules (§2.1: the decode set D_t and the prefill
+ * budget p_t; §3.1 caps p_t).  decode_seq_ids / decode_ctx_lens are HOST
+ * arrays of n_decodes entries: the page-table row of each decoding sequence
+ * and the number of tokens it has cached (its new token goes to position
+ * ctx; it attends ctx + 1 keys).  prefill_seq_id is the page-table row of the
+ * prompt being prefilled (ignored when p_t == 0); its chunk covers positions
+ * [chunk_start, chunk_start + p_t) and row j attends keys
+ * [0, chunk_start + j].  page_table and slots are DEVICE arrays. */
+typedef struct {
+    const int32_t *decode_seq_ids;  /* host  [n_decodes]                  */
+    const int32_t *decode_ctx_lens; /* host  [n_decodes]                  */
+    int32_t n_decodes;              /* |D_t| >= 0                         */
+    int32_t prefill_seq_id;         /* row of page_table, or -1           */
+    int32_t chunk_start;            /* first position of the chunk        */
+    int32_t p_t;                    /* chunk length, 0 = decode only      */
+    const int32_t *page_table;      /* device [num_seqs][max_pages_per_seq] */
+    const int32_t *slots;           /* device [n_decodes + p_t]           */
+} mx_iter_desc;
+
+/* Per-layer tensors of one iteration (all DEVICE pointers). */
+typedef struct {
+    const void *q;  /* [n_tokens][Hq][128]  */
+    const void *k;  /* [n_tokens][Hkv][128] */
+    const void *v;  /* [n_tokens][Hkv][128] */
+    void *k_pool;   /* [num_pages][Hkv][16][128] */
+    void *v_pool;   /* [num_pages][Hkv][16][128] */
+    void *out;      /* [n_tokens][Hq][128]  */
+} mx_layer_bufs;
+
+/* Create a context on CUDA device `device` (made current for the call) and
+ * allocate its fixed workspace.  *out receives the context.  Errors:
+ * MX_EINVAL (geometry), MX_EDEVICE (not an sm_100-family GPU), MX_ECUDA. */
+int mx_create(mx_ctx **out, const mx_geom *geom, int device);
+
+/* Free a context and its workspace (synchronises the device first).
+ * NULL is accepted. */
+int mx_destroy(mx_ctx *ctx);
+
+/* KV append (§2.1 PagedAttention; §3.2 KV layout unchanged): for each token
+ * t < n_tokens with slots[t] >= 0 and every KV head h, copy k[t][h][:] to
+ * k_pool[slots[t] / 16][h][slots[t] % 16][:] and likewise for v.  slots is a
+ * DEVICE array; the page table enters through it (slot =
+ * page_table[seq][pos / 16] * 16 + pos % 16).  Each slot must appear at most
+ * once.  Slots beyond the pool are skipped and flag MX_ERRBIT_SLOT.
+ * Asynchronous on `stream`. */
+int mx_kv_append(mx_ctx *ctx, const int32_t *slots, int32_t n_tokens,
+                 const void *k, const void *v, void *k_pool, void *v_pool,
+                 void *stream);
+
+/* One layer of the mixed iteration in ONE persistent kernel launch: the KV
+ * append of all n_decodes + p_t tokens plus causal paged GQA attention for
+ * every query row and head, written to out as bf16.  Decode rows use a
+ * split-KV flash-decode with a log-sum-exp merge; chunk rows use tcgen05
+ * tensor-core tiles.  Asynchronous on `stream`.  Errors: MX_EINVAL /
+ * MX_ECAPACITY (host validation, nothing launched), MX_ECUDA. */
+int mx_mixed_attention(mx_ctx *ctx, const mx_iter_desc *desc,
+                       const mx_layer_bufs *bufs, void *stream);
+
+/* A whole iteration: the same schedule `desc` run through n_layers layers
+ * (layers[l] holds layer l's tensors), one launch per layer.  Records CUDA
+ * events before the first and after the last launch, waits for the second,
+ * and stores the elapsed device time in microseconds in *device_us_out (the
+ * L_t of Eq. 1 as completed on the device).  Reads and clears the device
+ * error word: MX_ERANGE_PAGE / MX_ERANGE_SLOT / MX_ETIMEOUT if a kernel
+ * flagged one (the time is still stored). */
+int mx_iteration(mx_ctx *ctx, const mx_iter_desc *desc, int32_t n_layers,
+                 const mx_layer_bufs *layers, float *device_us_out,
+                 void *stream);
+
+/* Wait for `stream`, then read and clear the device error word. */
+int mx_sync_status(mx_ctx *ctx, void *stream);
+
+/* Copy a NUL-terminated description of the context's last failure into buf
+ * (at most len bytes).  Returns the length written, or MX_EINVAL. */
+int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
+
+/* Tunables.  MX_OPT_SPLIT_KEYS: keys per decode split (multiple of 128,
+ * 0 = automatic).  MX_OPT_GRID: persistent grid size (0 = number of SMs). */
+#define MX_OPT_SPLIT_KEYS 1
+#define MX_OPT_GRID 2
+int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
+
+/* Number of work items and decode split length chosen for the last planned
+ * call (for reporting). */
+int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
+                 int32_t *n_prefill_items);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MIXATTN_H */

@@ -1,0 +1,10 @@
+"""GB300-native mixed prefill/decode paged attention (the iteration observed
+by the Decode-Latency Feedback Prefill controller, arxiv 2609.38386).
+
+The compute runs in ``libmixattn.so`` (hand-written CUDA for sm_103a, C ABI in
+``include/mixattn.h``); this package is its ctypes binding plus the host-side
+DLFP controller.  Creating a Context (or calling ``load()``) without the built
+library raises ImportError: there is no fallback path.
+"""
+from ._binding import (EXPORTS, LIB_PATH, MX_OPT_GRID, MX_OPT_SPLIT_KEYS, Context,  # noqa: F401
+                       MxError, load)

@@ -1,0 +1,182 @@
+"""ctypes binding of libmixattn.so: argument marshalling only.
+
+Every step of the mixed iteration runs in the library's CUDA kernels; this
+module converts torch tensors / numpy arrays to pointers and return codes to
+exceptions.  If the library is missing the import fails loudly: there is no
+CPU path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libmixattn.so")
+
+MX_OK = 0
+ERRORS = {-1: "MX_EINVAL", -2: "MX_ERANGE_PAGE", -3: "MX_ERANGE_SLOT", -4: "MX_ECUDA",
+          -5: "MX_ETIMEOUT", -6: "MX_EDEVICE", -7: "MX_ECAPACITY"}
+MX_OPT_SPLIT_KEYS = 1
+MX_OPT_GRID = 2
+
+# Names every C-ABI build must export (the declarations of include/mixattn.h).
+EXPORTS = ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",
+           "mx_iteration", "mx_sync_status", "mx_error_detail", "mx_set_option",
+           "mx_last_plan")
+
+
+class MxError(RuntimeError):
+    def __init__(self, code, detail=""):
+        self.code = code
+        super().__init__(f"{ERRORS.get(code, code)}: {detail}")
+
+
+class mx_geom(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "num_q_heads", "num_kv_heads", "head_dim", "page_size", "num_pages",
+        "num_seqs", "max_pages_per_seq", "max_tokens", "max_decodes")]
+
+
+class mx_iter_desc(ctypes.Structure):
+    _fields_ = [("decode_seq_ids", ctypes.c_void_p), ("decode_ctx_lens", ctypes.c_void_p),
+                ("n_decodes", ctypes.c_int32), ("prefill_seq_id", ctypes.c_int32),
+                ("chunk_start", ctypes.c_int32), ("p_t", ctypes.c_int32),
+                ("page_table", ctypes.c_void_p), ("slots", ctypes.c_void_p)]
+
+
+class mx_layer_bufs(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("q", "k", "v", "k_pool", "v_pool", "out")]
+
+
+_lib = None
+
+
+def load():
+    """Load the in-tree library (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"{LIB_PATH} not found: build it with "
+                              "`python -c 'import __graft_entry__ as g; g.build()'`")
+        lib = ctypes.CDLL(LIB_PATH)
+        P, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+        sig = {
+            "mx_create": [ctypes.POINTER(P), ctypes.POINTER(mx_geom), ctypes.c_int],
+            "mx_destroy": [P],
+            "mx_kv_append": [P, P, i32, P, P, P, P, P],
+            "mx_mixed_attention": [P, ctypes.POINTER(mx_iter_desc),
+                                   ctypes.POINTER(mx_layer_bufs), P],
+            "mx_iteration": [P, ctypes.POINTER(mx_iter_desc), i32,
+                             ctypes.POINTER(mx_layer_bufs), ctypes.POINTER(ctypes.c_float), P],
+            "mx_sync_status": [P, P],
+            "mx_error_detail": [P, ctypes.c_char_p, i32],
+            "mx_set_option": [P, i32, i64],
+            "mx_last_plan": [P, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)],
+        }
+        for name, args in sig.items():
+            f = getattr(lib, name)
+            f.argtypes = args
+            f.restype = ctypes.c_int
+        _lib = lib
+    return _lib
+
+
+def _ptr(t):
+    """Device pointer of a torch tensor (or an int address, or None)."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream_handle(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+class Context:
+    """A mixattn context (fixed geometry and workspace) on one GPU."""
+
+    def __init__(self, *, num_q_heads, num_kv_heads=8, head_dim=128, page_size=16,
+                 num_pages, num_seqs, max_pages_per_seq, max_tokens, max_decodes,
+                 device=0):
+        self._lib = load()
+        self.geom = mx_geom(num_q_heads, num_kv_heads, head_dim, page_size, num_pages,
+                            num_seqs, max_pages_per_seq, max_tokens, max_decodes)
+        self.device = device
+        h = ctypes.c_void_p()
+        rc = self._lib.mx_create(ctypes.byref(h), ctypes.byref(self.geom), device)
+        if rc != MX_OK:
+            raise MxError(rc, "mx_create failed")
+        self._h = h
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._lib.mx_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _check(self, rc):
+        if rc != MX_OK:
+            buf = ctypes.create_string_buffer(512)
+            self._lib.mx_error_detail(self._h, buf, 512)
+            raise MxError(rc, buf.value.decode(errors="replace"))
+
+    # ------------------------------------------------------------------ calls
+    def set_option(self, option, value):
+        self._check(self._lib.mx_set_option(self._h, option, int(value)))
+
+    def last_plan(self):
+        a, b, c = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+        self._check(self._lib.mx_last_plan(self._h, ctypes.byref(a), ctypes.byref(b),
+                                           ctypes.byref(c)))
+        return {"n_items": a.value, "split_keys": b.value, "n_prefill_items": c.value}
+
+    def kv_append(self, slots, k, v, k_pool, v_pool, stream=None):
+        n = int(slots.shape[0])
+        self._check(self._lib.mx_kv_append(self._h, _ptr(slots), n, _ptr(k), _ptr(v),
+                                           _ptr(k_pool), _ptr(v_pool), _stream_handle(stream)))
+
+    def make_desc(self, *, decode_seq_ids, decode_ctx_lens, prefill_seq_id=-1,
+                  chunk_start=0, p_t=0, page_table, slots):
+        """Descriptor with HOST decode arrays and DEVICE page_table/slots.
+        The returned object keeps the host arrays alive."""
+        ids = np.ascontiguousarray(np.asarray(decode_seq_ids, dtype=np.int32))
+        lens = np.ascontiguousarray(np.asarray(decode_ctx_lens, dtype=np.int32))
+        d = mx_iter_desc(ids.ctypes.data if len(ids) else None,
+                         lens.ctypes.data if len(lens) else None, len(lens),
+                         int(prefill_seq_id), int(chunk_start), int(p_t),
+                         _ptr(page_table), _ptr(slots))
+        d._keep = (ids, lens)
+        return d
+
+    @staticmethod
+    def make_bufs(q, k, v, k_pool, v_pool, out):
+        return mx_layer_bufs(_ptr(q), _ptr(k), _ptr(v), _ptr(k_pool), _ptr(v_pool), _ptr(out))
+
+    def mixed_attention(self, desc, bufs, stream=None):
+        self._check(self._lib.mx_mixed_attention(self._h, ctypes.byref(desc),
+                                                 ctypes.byref(bufs), _stream_handle(stream)))
+
+    def iteration(self, desc, layers, stream=None):
+        """Run all layers; returns the device-completion time in microseconds."""
+        arr = (mx_layer_bufs * max(len(layers), 1))(*layers)
+        us = ctypes.c_float()
+        self._check(self._lib.mx_iteration(self._h, ctypes.byref(desc), len(layers), arr,
+                                           ctypes.byref(us), _stream_handle(stream)))
+        return float(us.value)
+
+    def sync_status(self, stream=None):
+        self._check(self._lib.mx_sync_status(self._h, _stream_handle(stream)))

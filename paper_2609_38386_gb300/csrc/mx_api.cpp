@@ -1,0 +1,638 @@
+// C-ABI of the mixed-iteration library: context, host validation, the
+// per-iteration planner (work list), TMA descriptors and launches.
+#include "../../include/mixattn.h"
+#include "mx_internal.h"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+namespace mx {
+cudaError_t init_layer_kernel();
+cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream);
+cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int num_pages,
+                             const uint16_t *k, const uint16_t *v, uint16_t *k_pool,
+                             uint16_t *v_pool, uint32_t *err, cudaStream_t stream);
+}  // namespace mx
+
+using namespace mx;
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+constexpr int kPlanSlots = 4;         // ring of work-list buffers
+constexpr int kPartSlots = 16384;     // split partials capacity
+constexpr int kMaxSplitKeys = kWarps * 32 * kPage;  // 4096: one page id per lane
+constexpr uint64_t kTimeoutNs = 1000000000ull;      // 1 s bound on in-kernel waits
+
+}  // namespace
+
+struct mx_ctx {
+    mx_geom g{};
+    int device = 0;
+    int num_sms = 0;
+    int max_items = 0;
+    // workspace (device)
+    uint8_t *ws = nullptr;
+    float *part_o = nullptr;
+    float *part_lse = nullptr;
+    uint32_t *merge_cnt = nullptr;
+    uint32_t *work_cnt = nullptr;
+    uint32_t *err = nullptr;
+    uint8_t *plan_dev[kPlanSlots] = {};
+    // pinned staging for the work list
+    uint8_t *plan_host[kPlanSlots] = {};
+    cudaEvent_t plan_ev[kPlanSlots] = {};
+    bool plan_ev_used[kPlanSlots] = {};
+    size_t plan_bytes = 0;
+    int plan_next = 0;
+    cudaEvent_t ev_start = nullptr, ev_end = nullptr;
+    EncodeTiledFn encode = nullptr;
+    // options
+    int split_keys_opt = 0;
+    int grid_opt = 0;
+    // last plan
+    int last_items = 0, last_split = 0, last_prefill_items = 0;
+    std::string last_error;
+};
+
+namespace {
+
+int fail(mx_ctx *c, int code, const char *fmt, ...)
+{
+    if (c) {
+        char buf[512];
+        va_list ap;
+        va_start(ap, fmt);
+        vsnprintf(buf, sizeof buf, fmt, ap);
+        va_end(ap);
+        c->last_error = buf;
+    }
+    return code;
+}
+
+int cuda_fail(mx_ctx *c, cudaError_t e, const char *what)
+{
+    return fail(c, MX_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct Plan {
+    int n_items = 0;
+    int n_prefill = 0;
+    int split_keys = 0;
+    int slot = 0;
+    const int4 *items_dev = nullptr;
+    const DecodeInfo *dec_dev = nullptr;
+};
+
+// Staging layout of one plan: DecodeInfo[n_decodes], then int4 items[n_items]
+// (both 16-byte records), uploaded with one copy.
+size_t plan_capacity_bytes(const mx_ctx *c)
+{
+    return (size_t)std::max(c->g.max_decodes, 1) * sizeof(DecodeInfo) + (size_t)c->max_items * sizeof(int4);
+}
+
+int validate(mx_ctx *c, const mx_iter_desc *d)
+{
+    if (!c || !d)
+        return fail(c, MX_EINVAL, "null context or descriptor");
+    const mx_geom &g = c->g;
+    if (d->n_decodes < 0 || d->p_t < 0 || d->chunk_start < 0)
+        return fail(c, MX_EINVAL, "negative n_decodes, p_t or chunk_start");
+    if (d->n_decodes > g.max_decodes)
+        return fail(c, MX_ECAPACITY, "n_decodes %d > max_decodes %d", d->n_decodes, g.max_decodes);
+    if ((int64_t)d->n_decodes + d->p_t > g.max_tokens)
+        return fail(c, MX_ECAPACITY, "n_decodes + p_t = %lld > max_tokens %d",
+                    (long long)d->n_decodes + d->p_t, g.max_tokens);
+    const int64_t cap = (int64_t)g.max_pages_per_seq * kPage;
+    if (d->n_decodes > 0 && (!d->decode_seq_ids || !d->decode_ctx_lens))
+        return fail(c, MX_EINVAL, "decode_seq_ids / decode_ctx_lens are null");
+    for (int i = 0; i < d->n_decodes; ++i) {
+        const int s = d->decode_seq_ids[i], n = d->decode_ctx_lens[i];
+        if (s < 0 || s >= g.num_seqs)
+            return fail(c, MX_EINVAL, "decode %d: seq id %d outside [0, %d)", i, s, g.num_seqs);
+        if (n < 0 || (int64_t)n + 1 > cap)
+            return fail(c, MX_ECAPACITY, "decode %d: ctx %d + 1 exceeds %lld page-table slots", i, n,
+                        (long long)cap);
+    }
+    if (d->p_t > 0) {
+        if (d->prefill_seq_id < 0 || d->prefill_seq_id >= g.num_seqs)
+            return fail(c, MX_EINVAL, "prefill seq id %d outside [0, %d)", d->prefill_seq_id, g.num_seqs);
+        if ((int64_t)d->chunk_start + d->p_t > cap)
+            return fail(c, MX_ECAPACITY, "chunk end %lld exceeds %lld page-table slots",
+                        (long long)d->chunk_start + d->p_t, (long long)cap);
+    }
+    if (d->n_decodes + d->p_t > 0 && (!d->page_table || !d->slots))
+        return fail(c, MX_EINVAL, "page_table / slots are null");
+    return MX_OK;
+}
+
+int validate_bufs(mx_ctx *c, const mx_layer_bufs *b, int n_tokens)
+{
+    if (!b)
+        return fail(c, MX_EINVAL, "null layer buffers");
+    if (n_tokens == 0)
+        return MX_OK;
+    const void *ps[] = {b->q, b->k, b->v, b->k_pool, b->v_pool, b->out};
+    for (const void *p : ps) {
+        if (!p)
+            return fail(c, MX_EINVAL, "a layer tensor pointer is null");
+        if (!aligned16(p))
+            return fail(c, MX_EINVAL, "a layer tensor pointer is not 16-byte aligned");
+    }
+    return MX_OK;
+}
+
+// a1: the per-iteration work list.  Prefill tiles first, heaviest (latest
+// rows, most keys) first; then decode splits, longest first.
+int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
+{
+    const mx_geom &g = c->g;
+    const int hkv = g.num_kv_heads, hq = g.num_q_heads;
+    const int nd = d->n_decodes;
+    int64_t total_keys = 0;
+    for (int i = 0; i < nd; ++i)
+        total_keys += (int64_t)d->decode_ctx_lens[i] + 1;
+    total_keys *= hkv;
+
+    int split = c->split_keys_opt;
+    if (split <= 0) {
+        const int64_t target_items = 2LL * c->num_sms;
+        int64_t s = (total_keys + target_items - 1) / std::max<int64_t>(target_items, 1);
+        s = (s + 127) / 128 * 128;
+        split = (int)std::min<int64_t>(std::max<int64_t>(s, 512), kMaxSplitKeys);
+    }
+    split = std::min(std::max(split / 128 * 128, 128), kMaxSplitKeys);
+    auto count_parts = [&](int sk) {
+        int64_t parts = 0;
+        for (int i = 0; i < nd; ++i) {
+            const int ns = (d->decode_ctx_lens[i] + 1 + sk - 1) / sk;
+            if (ns > 1)
+                parts += (int64_t)ns * hkv;
+        }
+        return parts;
+    };
+    while (count_parts(split) > kPartSlots && split < kMaxSplitKeys)
+        split = std::min(split * 2, kMaxSplitKeys);
+    if (count_parts(split) > kPartSlots)
+        return fail(c, MX_ECAPACITY, "decode splits exceed the partial workspace");
+
+    // staging slot: wait until its previous upload has been consumed
+    const int slot = c->plan_next;
+    c->plan_next = (slot + 1) % kPlanSlots;
+    if (c->plan_ev_used[slot]) {
+        cudaError_t e = cudaEventSynchronize(c->plan_ev[slot]);
+        if (e != cudaSuccess)
+            return cuda_fail(c, e, "cudaEventSynchronize(plan)");
+    }
+    uint8_t *host = c->plan_host[slot];
+    DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(host);
+    const size_t items_off = (size_t)nd * sizeof(DecodeInfo);
+    int4 *items = reinterpret_cast<int4 *>(host + items_off);
+
+    int n = 0;
+    const int n_qt = (d->p_t + kTileM - 1) / kTileM;
+    for (int t = n_qt - 1; t >= 0; --t)
+        for (int h = 0; h < hq; ++h)
+            items[n++] = make_int4(ITEM_PREFILL, t, h, 0);
+    const int n_prefill = n;
+
+    int part = 0;
+    struct DItem { int keys; int i, h, s; };
+    std::vector<DItem> ditems;
+    ditems.reserve(64);
+    for (int i = 0; i < nd; ++i) {
+        const int keys = d->decode_ctx_lens[i] + 1;
+        const int ns = (keys + split - 1) / split;
+        dec[i].seq = d->decode_seq_ids[i];
+        dec[i].ctx = d->decode_ctx_lens[i];
+        dec[i].n_splits = ns;
+        dec[i].part_base = ns > 1 ? part : 0;
+        if (ns > 1)
+            part += ns * hkv;
+        for (int h = 0; h < hkv; ++h)
+            for (int s = 0; s < ns; ++s)
+                ditems.push_back({std::min(split, keys - s * split), i, h, s});
+    }
+    if (n_prefill + (int)ditems.size() > c->max_items)
+        return fail(c, MX_ECAPACITY, "work list of %zu items exceeds capacity %d",
+                    n_prefill + ditems.size(), c->max_items);
+    std::stable_sort(ditems.begin(), ditems.end(),
+                     [](const DItem &a, const DItem &b) { return a.keys > b.keys; });
+    for (const DItem &x : ditems)
+        items[n++] = make_int4(ITEM_DECODE, x.i, x.h, x.s);
+
+    const size_t bytes = items_off + (size_t)n * sizeof(int4);
+    cudaError_t e = cudaMemcpyAsync(c->plan_dev[slot], host, bytes, cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "cudaMemcpyAsync(plan)");
+    e = cudaEventRecord(c->plan_ev[slot], stream);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventRecord(plan)");
+    c->plan_ev_used[slot] = true;
+
+    out->n_items = n;
+    out->n_prefill = n_prefill;
+    out->split_keys = split;
+    out->slot = slot;
+    out->items_dev = reinterpret_cast<const int4 *>(c->plan_dev[slot] + items_off);
+    out->dec_dev = reinterpret_cast<const DecodeInfo *>(c->plan_dev[slot]);
+    c->last_items = n;
+    c->last_split = split;
+    c->last_prefill_items = n_prefill;
+    return MX_OK;
+}
+
+int encode_map(mx_ctx *c, CUtensorMap *m, const void *base, int rank, const cuuint64_t *dims,
+               const cuuint64_t *strides_bytes, const cuuint32_t *box)
+{
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = c->encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
+                           const_cast<void *>(base), dims, strides_bytes, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(c, MX_ECUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+    return MX_OK;
+}
+
+int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const Plan &pl,
+                LayerParams *P)
+{
+    const mx_geom &g = c->g;
+    std::memset(P, 0, sizeof *P);
+    const int n_tok = d->n_decodes + d->p_t;
+    P->q = static_cast<const uint16_t *>(b->q);
+    P->k = static_cast<const uint16_t *>(b->k);
+    P->v = static_cast<const uint16_t *>(b->v);
+    P->k_pool = static_cast<uint16_t *>(b->k_pool);
+    P->v_pool = static_cast<uint16_t *>(b->v_pool);
+    P->out = static_cast<uint16_t *>(b->out);
+    P->page_table = d->page_table;
+    P->slots = d->slots;
+    P->items = pl.items_dev;
+    P->dec = pl.dec_dev;
+    P->part_o = c->part_o;
+    P->part_lse = c->part_lse;
+    P->merge_cnt = c->merge_cnt;
+    P->work_cnt = c->work_cnt;
+    P->err = c->err;
+    P->n_items = pl.n_items;
+    P->n_decodes = d->n_decodes;
+    P->prefill_seq = d->p_t > 0 ? d->prefill_seq_id : 0;
+    P->chunk_start = d->chunk_start;
+    P->p_t = d->p_t;
+    P->hq = g.num_q_heads;
+    P->hkv = g.num_kv_heads;
+    P->n_rep = g.num_q_heads / g.num_kv_heads;
+    P->num_pages = g.num_pages;
+    P->max_pages = g.max_pages_per_seq;
+    P->split_keys = pl.split_keys;
+    P->has_prefill = pl.n_prefill > 0 ? 1 : 0;
+    P->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
+    P->timeout_ns = kTimeoutNs;
+    if (P->has_prefill) {
+        const cuuint64_t hd = kHeadDim;
+        {
+            const cuuint64_t dims[3] = {hd, (cuuint64_t)g.num_q_heads, (cuuint64_t)n_tok};
+            const cuuint64_t str[2] = {hd * 2, hd * 2 * g.num_q_heads};
+            const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileM};
+            int rc = encode_map(c, &P->tm_q, b->q, 3, dims, str, box);
+            if (rc)
+                return rc;
+        }
+        {
+            const cuuint64_t dims[3] = {hd, (cuuint64_t)g.num_kv_heads, (cuuint64_t)n_tok};
+            const cuuint64_t str[2] = {hd * 2, hd * 2 * g.num_kv_heads};
+            const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileN};
+            int rc = encode_map(c, &P->tm_k, b->k, 3, dims, str, box);
+            if (!rc)
+                rc = encode_map(c, &P->tm_v, b->v, 3, dims, str, box);
+            if (rc)
+                return rc;
+        }
+        {
+            const cuuint64_t rows = (cuuint64_t)g.num_pages * g.num_kv_heads * kPage;
+            const cuuint64_t dims[2] = {hd, rows};
+            const cuuint64_t str[1] = {hd * 2};
+            const cuuint32_t box[2] = {64, (cuuint32_t)kPage};
+            int rc = encode_map(c, &P->tm_kpool, b->k_pool, 2, dims, str, box);
+            if (!rc)
+                rc = encode_map(c, &P->tm_vpool, b->v_pool, 2, dims, str, box);
+            if (rc)
+                return rc;
+        }
+    }
+    return MX_OK;
+}
+
+int grid_for(const mx_ctx *c, const Plan &pl)
+{
+    int grid = c->grid_opt > 0 ? c->grid_opt : c->num_sms;
+    return std::max(1, std::min(grid, pl.n_items));
+}
+
+int read_error_word(mx_ctx *c)
+{
+    uint32_t w = 0;
+    cudaError_t e = cudaMemcpy(&w, c->err, sizeof w, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "reading the error word");
+    if (w == 0)
+        return MX_OK;
+    e = cudaMemset(c->err, 0, sizeof(uint32_t));
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "clearing the error word");
+    if (w & ERR_TIMEOUT)
+        return fail(c, MX_ETIMEOUT, "a bounded in-kernel wait timed out (error word 0x%x)", w);
+    if (w & ERR_PAGE)
+        return fail(c, MX_ERANGE_PAGE, "a page id outside [0, num_pages) was read (error word 0x%x)", w);
+    return fail(c, MX_ERANGE_SLOT, "a slot outside the pool was skipped (error word 0x%x)", w);
+}
+
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev)
+    {
+        if (cudaGetDevice(&prev) == cudaSuccess && prev != dev)
+            cudaSetDevice(dev);
+        else
+            prev = -1;
+    }
+    ~DeviceGuard()
+    {
+        if (prev >= 0)
+            cudaSetDevice(prev);
+    }
+};
+
+}  // namespace
+
+extern "C" {
+
+int mx_create(mx_ctx **out, const mx_geom *g, int device)
+{
+    if (!out || !g)
+        return MX_EINVAL;
+    *out = nullptr;
+    if (g->head_dim != kHeadDim || g->page_size != kPage || g->num_kv_heads <= 0 ||
+        g->num_q_heads <= 0 || g->num_q_heads % g->num_kv_heads != 0 ||
+        g->num_q_heads / g->num_kv_heads > kMaxRep || g->num_pages <= 0 || g->num_seqs <= 0 ||
+        g->max_pages_per_seq <= 0 || g->max_tokens < 0 || g->max_decodes < 0 ||
+        (int64_t)g->num_pages * g->num_kv_heads * kPage > INT32_MAX)
+        return MX_EINVAL;
+    const int rep = g->num_q_heads / g->num_kv_heads;
+    if (rep & (rep - 1))
+        return MX_EINVAL;
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev)
+        return MX_EDEVICE;
+    DeviceGuard guard(device);
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, device) != cudaSuccess || prop.major != 10)
+        return MX_EDEVICE;
+
+    mx_ctx *c = new mx_ctx();
+    c->g = *g;
+    c->device = device;
+    c->num_sms = prop.multiProcessorCount;
+    const int max_prefill_items = ((g->max_tokens + kTileM - 1) / kTileM) * g->num_q_heads;
+    c->max_items = max_prefill_items + kPartSlots + std::max(g->max_decodes, 1) * g->num_kv_heads;
+
+    auto bail = [&](cudaError_t e, const char *what) {
+        std::string msg = std::string(what) + ": " + cudaGetErrorString(e);
+        mx_destroy(c);
+        (void)msg;
+        return MX_ECUDA;
+    };
+    cudaError_t e;
+    if ((e = init_layer_kernel()) != cudaSuccess)
+        return bail(e, "cudaFuncSetAttribute");
+
+    const size_t part_o_bytes = (size_t)kPartSlots * kMaxRep * kHeadDim * sizeof(float);
+    const size_t part_lse_bytes = (size_t)kPartSlots * kMaxRep * sizeof(float);
+    const size_t merge_bytes = (size_t)std::max(g->max_decodes, 1) * g->num_kv_heads * sizeof(uint32_t);
+    c->plan_bytes = plan_capacity_bytes(c);
+    const size_t plan_stride = (c->plan_bytes + 255) & ~size_t(255);
+    const size_t total = part_o_bytes + part_lse_bytes + ((merge_bytes + 255) & ~size_t(255)) +
+                         256 /*counters + err*/ + kPlanSlots * plan_stride;
+    if ((e = cudaMalloc(&c->ws, total)) != cudaSuccess)
+        return bail(e, "cudaMalloc(workspace)");
+    uint8_t *p = c->ws;
+    c->part_o = reinterpret_cast<float *>(p);
+    p += part_o_bytes;
+    c->part_lse = reinterpret_cast<float *>(p);
+    p += part_lse_bytes;
+    c->merge_cnt = reinterpret_cast<uint32_t *>(p);
+    p += (merge_bytes + 255) & ~size_t(255);
+    c->work_cnt = reinterpret_cast<uint32_t *>(p);
+    c->err = c->work_cnt + 4;
+    p += 256;
+    for (int s = 0; s < kPlanSlots; ++s) {
+        c->plan_dev[s] = p;
+        p += plan_stride;
+        if ((e = cudaMallocHost(&c->plan_host[s], c->plan_bytes)) != cudaSuccess)
+            return bail(e, "cudaMallocHost(plan)");
+        if ((e = cudaEventCreateWithFlags(&c->plan_ev[s], cudaEventDisableTiming)) != cudaSuccess)
+            return bail(e, "cudaEventCreate");
+    }
+    if ((e = cudaMemset(c->merge_cnt, 0, merge_bytes)) != cudaSuccess ||
+        (e = cudaMemset(c->work_cnt, 0, 256)) != cudaSuccess)
+        return bail(e, "cudaMemset(workspace)");
+    if ((e = cudaEventCreate(&c->ev_start)) != cudaSuccess ||
+        (e = cudaEventCreate(&c->ev_end)) != cudaSuccess)
+        return bail(e, "cudaEventCreate");
+
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) {
+        mx_destroy(c);
+        return MX_ECUDA;
+    }
+    c->encode = reinterpret_cast<EncodeTiledFn>(fn);
+    if ((e = cudaDeviceSynchronize()) != cudaSuccess)
+        return bail(e, "cudaDeviceSynchronize");
+    *out = c;
+    return MX_OK;
+}
+
+int mx_destroy(mx_ctx *c)
+{
+    if (!c)
+        return MX_OK;
+    DeviceGuard guard(c->device);
+    cudaDeviceSynchronize();
+    for (int s = 0; s < kPlanSlots; ++s) {
+        if (c->plan_host[s])
+            cudaFreeHost(c->plan_host[s]);
+        if (c->plan_ev[s])
+            cudaEventDestroy(c->plan_ev[s]);
+    }
+    if (c->ev_start)
+        cudaEventDestroy(c->ev_start);
+    if (c->ev_end)
+        cudaEventDestroy(c->ev_end);
+    if (c->ws)
+        cudaFree(c->ws);
+    delete c;
+    return MX_OK;
+}
+
+int mx_kv_append(mx_ctx *c, const int32_t *slots, int32_t n_tokens, const void *k, const void *v,
+                 void *k_pool, void *v_pool, void *stream)
+{
+    if (!c)
+        return MX_EINVAL;
+    if (n_tokens < 0)
+        return fail(c, MX_EINVAL, "n_tokens < 0");
+    if (n_tokens == 0)
+        return MX_OK;
+    if (!slots || !k || !v || !k_pool || !v_pool)
+        return fail(c, MX_EINVAL, "null pointer");
+    if (!aligned16(k) || !aligned16(v) || !aligned16(k_pool) || !aligned16(v_pool))
+        return fail(c, MX_EINVAL, "tensor pointers must be 16-byte aligned");
+    DeviceGuard guard(c->device);
+    cudaError_t e = launch_kv_append(slots, n_tokens, c->g.num_kv_heads, c->g.num_pages,
+                                     static_cast<const uint16_t *>(k), static_cast<const uint16_t *>(v),
+                                     static_cast<uint16_t *>(k_pool), static_cast<uint16_t *>(v_pool),
+                                     c->err, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "kv_append launch");
+    return MX_OK;
+}
+
+int mx_mixed_attention(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, void *stream)
+{
+    int rc = validate(c, d);
+    if (rc)
+        return rc;
+    const int n_tok = d->n_decodes + d->p_t;
+    if ((rc = validate_bufs(c, b, n_tok)))
+        return rc;
+    if (n_tok == 0)
+        return MX_OK;
+    DeviceGuard guard(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Plan pl;
+    if ((rc = plan(c, d, st, &pl)))
+        return rc;
+    LayerParams P;
+    if ((rc = make_params(c, d, b, pl, &P)))
+        return rc;
+    cudaError_t e = launch_mixed_layer(P, grid_for(c, pl), st);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "mixed_layer launch");
+    return MX_OK;
+}
+
+int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_layer_bufs *layers,
+                 float *device_us_out, void *stream)
+{
+    int rc = validate(c, d);
+    if (rc)
+        return rc;
+    if (n_layers < 0 || (n_layers > 0 && !layers) || !device_us_out)
+        return fail(c, MX_EINVAL, "bad n_layers / layers / device_us_out");
+    const int n_tok = d->n_decodes + d->p_t;
+    for (int l = 0; l < n_layers; ++l)
+        if ((rc = validate_bufs(c, layers + l, n_tok)))
+            return rc;
+    DeviceGuard guard(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Plan pl;
+    const bool work = n_tok > 0 && n_layers > 0;
+    if (work && (rc = plan(c, d, st, &pl)))
+        return rc;
+    // all descriptors are encoded before the timed region starts
+    std::vector<LayerParams> params(work ? n_layers : 0);
+    for (int l = 0; work && l < n_layers; ++l)
+        if ((rc = make_params(c, d, layers + l, pl, &params[l])))
+            return rc;
+    cudaError_t e = cudaEventRecord(c->ev_start, st);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventRecord(start)");
+    for (int l = 0; work && l < n_layers; ++l) {
+        e = launch_mixed_layer(params[l], grid_for(c, pl), st);
+        if (e != cudaSuccess)
+            return cuda_fail(c, e, "mixed_layer launch");
+    }
+    if ((e = cudaEventRecord(c->ev_end, st)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventRecord(end)");
+    if ((e = cudaEventSynchronize(c->ev_end)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventSynchronize(end)");
+    float ms = 0.f;
+    if ((e = cudaEventElapsedTime(&ms, c->ev_start, c->ev_end)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventElapsedTime");
+    *device_us_out = ms * 1000.0f;
+    return read_error_word(c);
+}
+
+int mx_sync_status(mx_ctx *c, void *stream)
+{
+    if (!c)
+        return MX_EINVAL;
+    DeviceGuard guard(c->device);
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "cudaStreamSynchronize");
+    return read_error_word(c);
+}
+
+int mx_error_detail(mx_ctx *c, char *buf, int32_t len)
+{
+    if (!c || !buf || len <= 0)
+        return MX_EINVAL;
+    const size_t n = std::min<size_t>(c->last_error.size(), (size_t)len - 1);
+    std::memcpy(buf, c->last_error.data(), n);
+    buf[n] = '\0';
+    return (int)n;
+}
+
+int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
+{
+    if (!c)
+        return MX_EINVAL;
+    switch (option) {
+    case MX_OPT_SPLIT_KEYS:
+        if (value < 0 || value > kMaxSplitKeys || value % 128)
+            return fail(c, MX_EINVAL, "split keys must be 0 or a multiple of 128 up to %d", kMaxSplitKeys);
+        c->split_keys_opt = (int)value;
+        return MX_OK;
+    case MX_OPT_GRID:
+        if (value < 0 || value > 65535)
+            return fail(c, MX_EINVAL, "grid must be in [0, 65535]");
+        c->grid_opt = (int)value;
+        return MX_OK;
+    default:
+        return fail(c, MX_EINVAL, "unknown option %d", option);
+    }
+}
+
+int mx_last_plan(mx_ctx *c, int32_t *n_items, int32_t *split_keys, int32_t *n_prefill_items)
+{
+    if (!c)
+        return MX_EINVAL;
+    if (n_items)
+        *n_items = c->last_items;
+    if (split_keys)
+        *split_keys = c->last_split;
+    if (n_prefill_items)
+        *n_prefill_items = c->last_prefill_items;
+    return MX_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,88 @@
+// Shared host/device definitions of the mixed-iteration kernels.
+#pragma once
+
+#include <cuda.h>
+#include <vector_types.h>
+
+#include <cstdint>
+
+namespace mx {
+
+constexpr int kHeadDim = 128;
+constexpr int kPage = 16;
+constexpr int kThreads = 256;            // 8 warps per CTA
+constexpr int kWarps = kThreads / 32;
+constexpr int kMaxRep = 8;               // Hq / Hkv supported up to 8
+
+// Prefill tile geometry: 128 query rows x 128 keys per tcgen05 tile.
+constexpr int kTileM = 128;
+constexpr int kTileN = 128;
+
+// Shared-memory plan (bytes, offsets from a 1024-aligned base).
+constexpr int kHalfTile = kTileM * 64 * 2;             // 128 rows x 64 bf16 = 16 KiB
+constexpr int kTileBytes = 2 * kHalfTile;              // 32 KiB
+constexpr int kSmemQ = 0;
+constexpr int kSmemK = kSmemQ + kTileBytes;            // 2 stages
+constexpr int kSmemV = kSmemK + 2 * kTileBytes;        // 2 stages
+constexpr int kSmemP = kSmemV + 2 * kTileBytes;        // 2 buffers
+constexpr int kSmemData = kSmemP + 2 * kTileBytes;     // 224 KiB
+constexpr int kSmemMisc = kSmemData;                   // barriers etc.
+constexpr int kSmemMiscBytes = 1024;
+constexpr int kSmemTotal = kSmemData + kSmemMiscBytes + 1024;  // + alignment slack
+
+// Decode ring: each warp owns kDecStages stages of one page (K 4 KiB + V 4 KiB).
+constexpr int kPageBytes = kPage * kHeadDim * 2;       // 4 KiB
+constexpr int kDecStageBytes = 2 * kPageBytes;         // 8 KiB
+constexpr int kDecStages = 3;
+static_assert(kWarps * kDecStages * kDecStageBytes <= kSmemData, "decode ring too large");
+
+constexpr uint32_t kTmemCols = 512;
+
+enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
+
+// Error bits (mirror MX_ERRBIT_* of the public header).
+constexpr uint32_t ERR_PAGE = 1u, ERR_SLOT = 2u, ERR_TIMEOUT = 4u;
+
+// Per-decode metadata uploaded with the work list.
+struct DecodeInfo {
+    int32_t seq;        // page-table row
+    int32_t ctx;        // cached tokens before this iteration
+    int32_t n_splits;   // splits of its key range [0, ctx]
+    int32_t part_base;  // first partial slot of (this decode, head 0)
+};
+
+struct LayerParams {
+    CUtensorMap tm_q;      // 3-D {128, Hq, n_tokens}, box {64, 1, 128}
+    CUtensorMap tm_k;      // 3-D {128, Hkv, n_tokens}, box {64, 1, 128}
+    CUtensorMap tm_v;
+    CUtensorMap tm_kpool;  // 2-D {128, num_pages*Hkv*16}, box {64, 16}
+    CUtensorMap tm_vpool;
+
+    const uint16_t *q, *k, *v;
+    uint16_t *k_pool, *v_pool, *out;
+
+    const int32_t *page_table;
+    const int32_t *slots;
+    const int4 *items;
+    const DecodeInfo *dec;
+
+    float *part_o;         // [slot][kMaxRep][128] normalised partial outputs
+    float *part_lse;       // [slot][kMaxRep] log2-sum-exp of each partial
+    uint32_t *merge_cnt;   // [max_decodes * Hkv] arrival counters (self-resetting)
+    uint32_t *work_cnt;    // [0] next item, [1] CTAs finished (self-resetting)
+    uint32_t *err;         // error word
+
+    int32_t n_items;
+    int32_t n_decodes;
+    int32_t prefill_seq;
+    int32_t chunk_start;
+    int32_t p_t;
+    int32_t hq, hkv, n_rep;
+    int32_t num_pages, max_pages;
+    int32_t split_keys;    // keys per decode split (multiple of 128)
+    int32_t has_prefill;   // allocate TMEM only when prefill tiles exist
+    float scale_log2;      // log2(e) / sqrt(head_dim)
+    uint64_t timeout_ns;   // bound on every in-kernel wait
+};
+
+}  // namespace mx

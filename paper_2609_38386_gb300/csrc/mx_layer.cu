@@ -1,0 +1,782 @@
+// One layer of the mixed prefill/decode iteration in one persistent launch.
+//
+// Semantics (paper §2.1, Eq. 1 setting; §3.2 attention and KV layout
+// unchanged): the |D_t| decode tokens and the p_t chunk tokens of one prompt
+// append their K/V to their page slots and attend causally over the paged
+// cache.  Query head h reads KV head h / (Hq / Hkv); scores are scaled by
+// 1/sqrt(128); a decode with ctx cached tokens sees ctx + 1 keys; chunk row j
+// sees keys [0, chunk_start + j].
+//
+// Work items (built on the host, fetched with one atomic counter):
+//   ITEM_PREFILL {t, hq}:   128 chunk rows [128t, 128t+128) of query head hq
+//                           against every visible key, on tcgen05 tensor cores
+//                           (S and O accumulators in TMEM), with the append
+//                           of the tile's K/V done by the head group's first
+//                           query head.
+//   ITEM_DECODE  {i, h, s}: split s of decode i's keys for KV head h, all n_rep
+//                           query heads of the group at once: a split-KV
+//                           flash-decode whose partial (O, lse) is merged by
+//                           the last-arriving split (no waiting).
+// New keys/values are read from the k/v inputs, never from the pages being
+// written in the same launch, so the append needs no ordering.
+#include "mx_internal.h"
+#include "mx_ptx.cuh"
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+namespace mx {
+
+struct Misc {
+    uint64_t bar_q;
+    uint64_t bar_kfull[2];
+    uint64_t bar_vfull[2];
+    uint64_t bar_kvempty[2];
+    uint64_t bar_sfull[2];
+    uint64_t bar_pfull[2];
+    uint64_t bar_odone[2];
+    uint32_t tmem_base;
+    int32_t item_idx[2];
+    int32_t abort;
+    int32_t last;
+};
+static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
+
+// Instruction descriptors: S = Q K^T (both K-major) and O = P V (V MN-major).
+constexpr uint32_t kIdescS = idesc_bf16_f32(128, 128, false, false);
+constexpr uint32_t kIdescO = idesc_bf16_f32(128, 128, false, true);
+constexpr uint32_t kSwz128 = 2;
+
+__device__ __forceinline__ void flag_error(const LayerParams &P, uint32_t bit)
+{
+    atomicOr(P.err, bit);
+}
+
+__device__ __forceinline__ void set_abort(const LayerParams &P, Misc *misc)
+{
+    *(volatile int32_t *)&misc->abort = 1;
+    flag_error(P, ERR_TIMEOUT);
+}
+
+__device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
+
+// ---------------------------------------------------------------------------
+// Decode split: keys [k_lo, k_hi) of decode di, KV head h.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t stage,
+                                                  int pid, int kb, int n, int k_hi, int di,
+                                                  int h, int lane)
+{
+    const uint16_t *kin = P.k + ((size_t)di * P.hkv + h) * kHeadDim;
+    const uint16_t *vin = P.v + ((size_t)di * P.hkv + h) * kHeadDim;
+    const size_t pbase = ((size_t)(pid < 0 ? 0 : pid) * P.hkv + h) * kPage * kHeadDim;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const int ci = lane + 32 * e;  // 16-byte chunk of the 16 x 256 B page tile
+        const int row = ci >> 4, c = ci & 15;
+        const int key = kb + row;
+        const uint16_t *ks, *vs;
+        uint32_t bytes = key < k_hi ? 16u : 0u;
+        if (key < n) {
+            ks = P.k_pool + pbase + row * kHeadDim + c * 8;
+            vs = P.v_pool + pbase + row * kHeadDim + c * 8;
+            if (pid < 0)
+                bytes = 0;
+        } else {
+            ks = kin + c * 8;  // key == n: the decode's own new key
+            vs = vin + c * 8;
+            if (key != n)
+                bytes = 0;
+        }
+        const uint32_t dst = stage + row * 256 + ((c ^ (row & 7)) << 4);
+        cp_async16(dst, ks, bytes);
+        cp_async16(dst + kPageBytes, vs, bytes);
+    }
+}
+
+__device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int di, int h,
+                            int s)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const DecodeInfo D = P.dec[di];
+    const int n = D.ctx;
+    const int nrep = P.n_rep;
+    const int k_lo = s * P.split_keys;
+    const int k_hi = min(k_lo + P.split_keys, n + 1);
+    const int pg_lo = k_lo / kPage;
+    const int npg = (k_hi - k_lo + kPage - 1) / kPage;
+    const int g = lane >> 2, tq = lane & 3;
+
+    // The split holding the new key appends it (each slot written once).
+    if (s == D.n_splits - 1 && warp == 0) {
+        const int slot = P.slots[di];
+        if (slot >= 0) {
+            if (slot >= P.num_pages * kPage) {
+                if (lane == 0)
+                    flag_error(P, ERR_SLOT);
+            } else {
+                const size_t dst = (((size_t)(slot / kPage) * P.hkv + h) * kPage + slot % kPage) * kHeadDim;
+                const size_t src = ((size_t)di * P.hkv + h) * kHeadDim;
+                const int c = lane & 15;
+                if (lane < 16)
+                    reinterpret_cast<uint4 *>(P.k_pool + dst)[c] =
+                        __ldg(reinterpret_cast<const uint4 *>(P.k + src) + c);
+                else
+                    reinterpret_cast<uint4 *>(P.v_pool + dst)[c] =
+                        __ldg(reinterpret_cast<const uint4 *>(P.v + src) + c);
+            }
+        }
+    }
+
+    // Q^T fragments (B operand of S^T = K Q^T): query row g of the group.
+    uint32_t qb[8][2];
+    {
+        const uint16_t *qrow = P.q + ((size_t)di * P.hq + h * nrep + (g < nrep ? g : 0)) * kHeadDim;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+            if (g < nrep) {
+                qb[kk][0] = __ldg(reinterpret_cast<const uint32_t *>(qrow + kk * 16 + 2 * tq));
+                qb[kk][1] = __ldg(reinterpret_cast<const uint32_t *>(qrow + kk * 16 + 8 + 2 * tq));
+            } else {
+                qb[kk][0] = qb[kk][1] = 0u;
+            }
+        }
+    }
+
+    // This warp's pages: local indices warp, warp + 8, ...
+    const int my_n = npg > warp ? (npg - warp + kWarps - 1) / kWarps : 0;
+    int pid_l = -1;
+    if (lane < my_n) {
+        const int lp = pg_lo + warp + kWarps * lane;
+        if (lp * kPage < n) {  // pages holding cached keys only
+            int pid = __ldg(P.page_table + (size_t)D.seq * P.max_pages + lp);
+            if (pid < 0 || pid >= P.num_pages) {
+                flag_error(P, ERR_PAGE);
+                pid = -1;
+            }
+            pid_l = pid;
+        }
+    }
+
+    const uint32_t ring = smem_u32(smem) + warp * (kDecStages * kDecStageBytes);
+    float acc[8][4];
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt)
+        acc[mt][0] = acc[mt][1] = acc[mt][2] = acc[mt][3] = 0.f;
+    float m0 = neg_inf(), m1 = neg_inf(), l0 = 0.f, l1 = 0.f;
+    const float sl = P.scale_log2;
+
+#pragma unroll
+    for (int k = 0; k < kDecStages - 1; ++k) {
+        const int pid = __shfl_sync(0xffffffffu, pid_l, k & 31);
+        if (k < my_n)
+            decode_issue_page(P, ring + k * kDecStageBytes, pid,
+                              (pg_lo + warp + kWarps * k) * kPage, n, k_hi, di, h, lane);
+        cp_async_commit();
+    }
+
+    for (int k = 0; k < my_n; ++k) {
+        {
+            const int kn = k + kDecStages - 1;
+            const int pid = __shfl_sync(0xffffffffu, pid_l, kn & 31);
+            if (kn < my_n)
+                decode_issue_page(P, ring + (kn % kDecStages) * kDecStageBytes, pid,
+                                  (pg_lo + warp + kWarps * kn) * kPage, n, k_hi, di, h, lane);
+            cp_async_commit();
+        }
+        cp_async_wait<kDecStages - 1>();
+        __syncwarp();
+
+        const uint32_t kbase = ring + (k % kDecStages) * kDecStageBytes;
+        const uint32_t vbase = kbase + kPageBytes;
+        const int kb = (pg_lo + warp + kWarps * k) * kPage;
+        const int nv = min(kPage, k_hi - kb);  // valid keys in this page (>= 1)
+
+        // S^T (16 keys x 8 query rows) = K (16 x 128) * Q^T (128 x 8)
+        float sc[4] = {0.f, 0.f, 0.f, 0.f};
+        {
+            const int mi = lane >> 3;
+            const int row = (lane & 7) + (mi & 1) * 8;
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+                const int chunk = kk * 2 + (mi >> 1);
+                uint32_t a0, a1, a2, a3;
+                ldsm_x4(kbase + row * 256 + ((chunk ^ (row & 7)) << 4), a0, a1, a2, a3);
+                mma_bf16_16816(sc, a0, a1, a2, a3, qb[kk][0], qb[kk][1]);
+            }
+        }
+        // online softmax over this page's keys (log2 domain), per query column
+        const float x0 = g < nv ? sc[0] * sl : neg_inf();
+        const float x1 = g < nv ? sc[1] * sl : neg_inf();
+        const float x2 = g + 8 < nv ? sc[2] * sl : neg_inf();
+        const float x3 = g + 8 < nv ? sc[3] * sl : neg_inf();
+        float mx0 = fmaxf(x0, x2), mx1 = fmaxf(x1, x3);
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+        }
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+        const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
+        const float p0 = ex2(x0 - mn0), p1 = ex2(x1 - mn1);
+        const float p2 = ex2(x2 - mn0), p3 = ex2(x3 - mn1);
+        l0 = l0 * al0 + p0 + p2;
+        l1 = l1 * al1 + p1 + p3;
+        m0 = mn0;
+        m1 = mn1;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+            acc[mt][0] *= al0;
+            acc[mt][1] *= al1;
+            acc[mt][2] *= al0;
+            acc[mt][3] *= al1;
+        }
+        // P^T as the B operand (keys x query rows): transpose the 8x8 blocks
+        const uint32_t b0 = movmatrix_t(pack_bf16(p0, p1));
+        const uint32_t b1 = movmatrix_t(pack_bf16(p2, p3));
+        // O^T (128 d x 8 rows) += V^T (128 x 16 keys) * P^T (16 x 8)
+        {
+            const int mi = lane >> 3;
+            const int key = (lane & 7) + (mi >> 1) * 8;
+#pragma unroll
+            for (int mt = 0; mt < 8; ++mt) {
+                const int chunk = mt * 2 + (mi & 1);
+                uint32_t a0, a1, a2, a3;
+                ldsm_x4_t(vbase + key * 256 + ((chunk ^ (key & 7)) << 4), a0, a1, a2, a3);
+                mma_bf16_16816(acc[mt], a0, a1, a2, a3, b0, b1);
+            }
+        }
+        __syncwarp();
+    }
+    cp_async_wait<0>();
+
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+        l0 += __shfl_xor_sync(0xffffffffu, l0, o);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+    }
+
+    // ---- combine the 8 warps of the CTA (shared memory)
+    __syncthreads();
+    float *so = reinterpret_cast<float *>(smem);               // [warp][8][128]
+    float *sml = so + kWarps * kMaxRep * kHeadDim;              // [warp][8][2]
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) {
+        const int d = mt * 16 + g;
+        so[(warp * kMaxRep + 2 * tq) * kHeadDim + d] = acc[mt][0];
+        so[(warp * kMaxRep + 2 * tq + 1) * kHeadDim + d] = acc[mt][1];
+        so[(warp * kMaxRep + 2 * tq) * kHeadDim + d + 8] = acc[mt][2];
+        so[(warp * kMaxRep + 2 * tq + 1) * kHeadDim + d + 8] = acc[mt][3];
+    }
+    if (g == 0) {
+        sml[(warp * kMaxRep + 2 * tq) * 2 + 0] = m0;
+        sml[(warp * kMaxRep + 2 * tq) * 2 + 1] = l0;
+        sml[(warp * kMaxRep + 2 * tq + 1) * 2 + 0] = m1;
+        sml[(warp * kMaxRep + 2 * tq + 1) * 2 + 1] = l1;
+    }
+    __syncthreads();
+
+    const int nsp = D.n_splits;
+    const int pslot = D.part_base + h * nsp + s;
+    for (int e = tid; e < nrep * kHeadDim; e += kThreads) {
+        const int q = e / kHeadDim, d = e % kHeadDim;
+        float M = neg_inf();
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w)
+            M = fmaxf(M, sml[(w * kMaxRep + q) * 2]);
+        float L = 0.f, O = 0.f;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) {
+            const float f = ex2(sml[(w * kMaxRep + q) * 2] - M);
+            L += f * sml[(w * kMaxRep + q) * 2 + 1];
+            O += f * so[(w * kMaxRep + q) * kHeadDim + d];
+        }
+        const float res = O / L;
+        if (nsp == 1) {
+            __nv_bfloat16 b = __float2bfloat16_rn(res);
+            P.out[((size_t)di * P.hq + h * nrep + q) * kHeadDim + d] =
+                *reinterpret_cast<uint16_t *>(&b);
+        } else {
+            P.part_o[((size_t)pslot * kMaxRep + q) * kHeadDim + d] = res;
+            if (d == 0) {
+                float lg;
+                asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(lg) : "f"(L));
+                P.part_lse[(size_t)pslot * kMaxRep + q] = M + lg;
+            }
+        }
+    }
+    if (nsp == 1)
+        return;
+
+    // ---- cross-split merge by the last-arriving split (no waiting)
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) {
+        const uint32_t prev = atomicAdd(P.merge_cnt + di * P.hkv + h, 1u);
+        misc->last = (prev == (uint32_t)(nsp - 1)) ? 1 : 0;
+    }
+    __syncthreads();
+    if (!misc->last)
+        return;
+    __threadfence();
+    const int base = D.part_base + h * nsp;
+    for (int e = tid; e < nrep * kHeadDim; e += kThreads) {
+        const int q = e / kHeadDim, d = e % kHeadDim;
+        float M = neg_inf();
+        for (int sp = 0; sp < nsp; ++sp)
+            M = fmaxf(M, __ldcg(P.part_lse + (size_t)(base + sp) * kMaxRep + q));
+        float W = 0.f, O = 0.f;
+        for (int sp = 0; sp < nsp; ++sp) {
+            const float f = ex2(__ldcg(P.part_lse + (size_t)(base + sp) * kMaxRep + q) - M);
+            W += f;
+            O += f * __ldcg(P.part_o + ((size_t)(base + sp) * kMaxRep + q) * kHeadDim + d);
+        }
+        __nv_bfloat16 b = __float2bfloat16_rn(O / W);
+        P.out[((size_t)di * P.hq + h * nrep + q) * kHeadDim + d] = *reinterpret_cast<uint16_t *>(&b);
+    }
+    if (tid == 0)
+        P.merge_cnt[di * P.hkv + h] = 0u;
+}
+
+// ---------------------------------------------------------------------------
+// Prefill tile: rows [128t, 128t + 128) of the chunk, query head hq.
+// Key tiles: nA paged tiles covering [0, chunk_start), then t + 1 tiles of
+// the chunk's own keys read from the k/v inputs.
+// ---------------------------------------------------------------------------
+__device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem,
+                             int t, int hq, uint32_t tile0, uint32_t item_no)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int kvh = hq / P.n_rep;
+    const int cs = P.chunk_start, p = P.p_t, nd = P.n_decodes;
+    const int nA = (cs + kTileN - 1) / kTileN;
+    const int nT = nA + t + 1;
+    const uint32_t sbase = smem_u32(smem);
+    const uint32_t sQ = sbase + kSmemQ, sK = sbase + kSmemK, sV = sbase + kSmemV,
+                   sP = sbase + kSmemP;
+    const uint32_t bar_q = smem_u32(&misc->bar_q);
+    volatile int *abort = &misc->abort;
+    const uint64_t tmo = P.timeout_ns;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            fence_proxy_async_smem();
+            mbar_expect_tx(bar_q, kTileBytes);
+            tma_load_3d(sQ, &P.tm_q, bar_q, 0, hq, nd + kTileM * t);
+            tma_load_3d(sQ + kHalfTile, &P.tm_q, bar_q, 64, hq, nd + kTileM * t);
+        }
+        const int oob_row = P.num_pages * P.hkv * kPage;
+        for (int i = 0; i < nT; ++i) {
+            const uint32_t c = tile0 + i;
+            const int st = c & 1;
+            const uint32_t ph = (c >> 1) & 1;
+            const bool paged = i < nA;
+            int pid_l = -1;
+            if (paged && lane < 8) {
+                const int lp = i * 8 + lane;
+                if (lp * kPage < cs) {
+                    int pid = __ldg(P.page_table + (size_t)P.prefill_seq * P.max_pages + lp);
+                    if (pid < 0 || pid >= P.num_pages) {
+                        flag_error(P, ERR_PAGE);
+                        pid = -1;
+                    }
+                    pid_l = pid;
+                }
+            }
+            int pids[8];
+#pragma unroll
+            for (int pg = 0; pg < 8; ++pg)
+                pids[pg] = __shfl_sync(0xffffffffu, pid_l, pg);
+            int ok = 1;
+            if (lane == 0) {
+                if (!mbar_wait(smem_u32(&misc->bar_kvempty[st]), ph ^ 1, abort, tmo)) {
+                    set_abort(P, misc);
+                    ok = 0;
+                }
+            }
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok)
+                break;
+            if (lane == 0) {
+                const uint32_t kf = smem_u32(&misc->bar_kfull[st]);
+                const uint32_t vf = smem_u32(&misc->bar_vfull[st]);
+                const uint32_t dk = sK + st * kTileBytes, dv = sV + st * kTileBytes;
+                mbar_expect_tx(kf, kTileBytes);
+                mbar_expect_tx(vf, kTileBytes);
+                if (paged) {
+#pragma unroll
+                    for (int pg = 0; pg < 8; ++pg) {
+                        const int y = pids[pg] >= 0 ? (pids[pg] * P.hkv + kvh) * kPage : oob_row;
+#pragma unroll
+                        for (int hf = 0; hf < 2; ++hf)
+                            tma_load_2d(dk + hf * kHalfTile + pg * 2048, &P.tm_kpool, kf, hf * 64, y);
+                    }
+#pragma unroll
+                    for (int pg = 0; pg < 8; ++pg) {
+                        const int y = pids[pg] >= 0 ? (pids[pg] * P.hkv + kvh) * kPage : oob_row;
+#pragma unroll
+                        for (int hf = 0; hf < 2; ++hf)
+                            tma_load_2d(dv + hf * kHalfTile + pg * 2048, &P.tm_vpool, vf, hf * 64, y);
+                    }
+                } else {
+                    const int z = nd + kTileN * (i - nA);
+#pragma unroll
+                    for (int hf = 0; hf < 2; ++hf)
+                        tma_load_3d(dk + hf * kHalfTile, &P.tm_k, kf, hf * 64, kvh, z);
+#pragma unroll
+                    for (int hf = 0; hf < 2; ++hf)
+                        tma_load_3d(dv + hf * kHalfTile, &P.tm_v, vf, hf * 64, kvh, z);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            bool ok = mbar_wait(bar_q, item_no & 1, abort, tmo);
+            tc_fence_after();
+            auto issue_pv = [&](int i) -> bool {
+                const uint32_t c = tile0 + i;
+                const int st = c & 1;
+                const uint32_t ph = (c >> 1) & 1;
+                if (!mbar_wait(smem_u32(&misc->bar_pfull[c & 1]), (c >> 1) & 1, abort, tmo))
+                    return false;
+                if (!mbar_wait(smem_u32(&misc->bar_vfull[st]), ph, abort, tmo))
+                    return false;
+                const uint32_t dv = sV + st * kTileBytes;
+                if (i == nA - 1 && (cs % kTileN) != 0) {
+                    // keys [cs, end of that page) of the last paged tile are not
+                    // cached yet: clear their value rows (later pages are zero).
+                    const int r0 = cs - i * kTileN;
+                    const int r1 = min(kTileN, (r0 + kPage - 1) / kPage * kPage);
+                    for (int r = r0; r < r1; ++r)
+                        for (int hf = 0; hf < 2; ++hf)
+                            for (int cc = 0; cc < 8; ++cc)
+                                asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(
+                                                 dv + hf * kHalfTile + r * 128 + cc * 16),
+                                             "r"(0u)
+                                             : "memory");
+                    fence_proxy_async_smem();
+                }
+                tc_fence_after();
+                const uint32_t pb = sP + (c & 1) * kTileBytes;
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint64_t a = smem_desc(pb + (kk >> 2) * kHalfTile + (kk & 3) * 32, 16, 1024, kSwz128);
+                    const uint64_t b = smem_desc(dv + kk * 2048, kHalfTile, 1024, kSwz128);
+                    tc_mma_ss(tmem + 256, a, b, kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
+                }
+                tc_commit(smem_u32(&misc->bar_odone[c & 1]));
+                tc_commit(smem_u32(&misc->bar_kvempty[st]));
+                return true;
+            };
+            for (int i = 0; ok && i < nT; ++i) {
+                const uint32_t c = tile0 + i;
+                const int st = c & 1;
+                const uint32_t ph = (c >> 1) & 1;
+                if (!mbar_wait(smem_u32(&misc->bar_kfull[st]), ph, abort, tmo)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t dk = sK + st * kTileBytes;
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint64_t a = smem_desc(sQ + (kk >> 2) * kHalfTile + (kk & 3) * 32, 16, 1024, kSwz128);
+                    const uint64_t b = smem_desc(dk + (kk >> 2) * kHalfTile + (kk & 3) * 32, 16, 1024, kSwz128);
+                    tc_mma_ss(tmem + (c & 1) * 128, a, b, kIdescS, kk > 0 ? 1u : 0u);
+                }
+                tc_commit(smem_u32(&misc->bar_sfull[c & 1]));
+                if (i > 0 && !issue_pv(i - 1))
+                    ok = false;
+            }
+            if (ok && !issue_pv(nT - 1))
+                ok = false;
+            if (!ok)
+                set_abort(P, misc);
+        }
+        __syncwarp();
+    } else if (warp < 4) {
+        // ------------------------------------------------ chunk KV append
+        if (hq % P.n_rep == 0) {
+            const int j0 = kTileM * t;
+            const int ntok = min(kTileM, p - j0);
+            for (int e = (warp - 2) * 32 + lane; e < ntok * 32; e += 64) {
+                const int tok = nd + j0 + e / 32, w = e % 32;
+                const int slot = __ldg(P.slots + tok);
+                if (slot < 0)
+                    continue;
+                if (slot >= P.num_pages * kPage) {
+                    flag_error(P, ERR_SLOT);
+                    continue;
+                }
+                const size_t dst = (((size_t)(slot / kPage) * P.hkv + kvh) * kPage + slot % kPage) * kHeadDim;
+                const size_t src = ((size_t)tok * P.hkv + kvh) * kHeadDim;
+                if (w < 16)
+                    reinterpret_cast<uint4 *>(P.k_pool + dst)[w] =
+                        __ldg(reinterpret_cast<const uint4 *>(P.k + src) + w);
+                else
+                    reinterpret_cast<uint4 *>(P.v_pool + dst)[w - 16] =
+                        __ldg(reinterpret_cast<const uint4 *>(P.v + src) + (w - 16));
+            }
+        }
+    } else {
+        // ------------------------------------------------ softmax / epilogue
+        const int q4 = warp - 4;
+        const int r = q4 * 32 + lane;          // tile row = TMEM lane
+        const int j = kTileM * t + r;          // chunk row offset
+        const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
+        const float sl = P.scale_log2;
+        float m_run = neg_inf(), l_run = 0.f;
+        bool ok = true;
+        for (int i = 0; i < nT; ++i) {
+            const uint32_t c = tile0 + i;
+            const int sb = c & 1;
+            if (!mbar_wait(smem_u32(&misc->bar_sfull[sb]), (c >> 1) & 1, abort, tmo)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            uint32_t sv[128];
+#pragma unroll
+            for (int gq = 0; gq < 4; ++gq)
+                tmem_ld32(tl + sb * 128 + 32 * gq, *reinterpret_cast<uint32_t(*)[32]>(&sv[32 * gq]));
+            tmem_wait_ld();
+            const int nvalid = i < nA ? min(kTileN, cs - i * kTileN)
+                                      : min(kTileN, j - kTileN * (i - nA) + 1);
+            float mx = neg_inf();
+#pragma unroll
+            for (int cc = 0; cc < 128; ++cc) {
+                const float x = cc < nvalid ? __uint_as_float(sv[cc]) * sl : neg_inf();
+                sv[cc] = __float_as_uint(x);
+                mx = fmaxf(mx, x);
+            }
+            const float m_new = fmaxf(m_run, mx);
+            const bool rescale = m_new > m_run + 8.0f;
+            const float m_use = rescale ? m_new : m_run;
+            float rs = 0.f;
+            uint32_t pk[64];
+#pragma unroll
+            for (int cc = 0; cc < 64; ++cc) {
+                const float e0 = ex2(__uint_as_float(sv[2 * cc]) - m_use);
+                const float e1 = ex2(__uint_as_float(sv[2 * cc + 1]) - m_use);
+                rs += e0 + e1;
+                pk[cc] = pack_bf16(e0, e1);
+            }
+            // P buffer (c & 1) was last read by tile c - 2's PV.
+            if (i >= 2 && !mbar_wait(smem_u32(&misc->bar_odone[c & 1]), ((c - 2) >> 1) & 1, abort, tmo)) {
+                ok = false;
+                break;
+            }
+            if (rescale && i > 0) {
+                // O must be stable: tile c - 1's PV has completed.
+                if (!mbar_wait(smem_u32(&misc->bar_odone[(c - 1) & 1]), ((c - 1) >> 1) & 1, abort, tmo)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const float alpha = ex2(m_run - m_use);
+#pragma unroll
+                for (int gq = 0; gq < 4; ++gq) {
+                    uint32_t o[32];
+                    tmem_ld32(tl + 256 + 32 * gq, o);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int x = 0; x < 32; ++x)
+                        o[x] = __float_as_uint(__uint_as_float(o[x]) * alpha);
+                    tmem_st32(tl + 256 + 32 * gq, o);
+                }
+                tmem_wait_st();
+                l_run *= alpha;
+            }
+            l_run += rs;
+            m_run = m_use;
+            // P row r into the 128-byte-swizzled K-major tile
+            const uint32_t prow = sP + (c & 1) * kTileBytes + r * 128;
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc) {
+                    const int w0 = hf * 32 + cc * 4;
+                    asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(
+                                     prow + hf * kHalfTile + ((cc ^ (r & 7)) << 4)),
+                                 "r"(pk[w0]), "r"(pk[w0 + 1]), "r"(pk[w0 + 2]), "r"(pk[w0 + 3])
+                                 : "memory");
+                }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(smem_u32(&misc->bar_pfull[c & 1]));
+        }
+        if (ok) {
+            const uint32_t cl = tile0 + nT - 1;
+            if (!mbar_wait(smem_u32(&misc->bar_odone[cl & 1]), (cl >> 1) & 1, abort, tmo))
+                ok = false;
+        }
+        if (!ok) {
+            set_abort(P, misc);
+        } else {
+            tc_fence_after();
+            const float inv = 1.0f / l_run;
+            uint16_t *orow = P.out + ((size_t)(nd + j) * P.hq + hq) * kHeadDim;
+#pragma unroll
+            for (int gq = 0; gq < 4; ++gq) {
+                uint32_t o[32];
+                tmem_ld32(tl + 256 + 32 * gq, o);
+                tmem_wait_ld();
+                if (j < p) {
+#pragma unroll
+                    for (int x = 0; x < 4; ++x) {
+                        uint4 v4;
+                        v4.x = pack_bf16(__uint_as_float(o[8 * x + 0]) * inv, __uint_as_float(o[8 * x + 1]) * inv);
+                        v4.y = pack_bf16(__uint_as_float(o[8 * x + 2]) * inv, __uint_as_float(o[8 * x + 3]) * inv);
+                        v4.z = pack_bf16(__uint_as_float(o[8 * x + 4]) * inv, __uint_as_float(o[8 * x + 5]) * inv);
+                        v4.w = pack_bf16(__uint_as_float(o[8 * x + 6]) * inv, __uint_as_float(o[8 * x + 7]) * inv);
+                        reinterpret_cast<uint4 *>(orow + 32 * gq)[x] = v4;
+                    }
+                }
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_constant__ LayerParams P)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    Misc *misc = reinterpret_cast<Misc *>(smem + kSmemMisc);
+    const int tid = threadIdx.x, warp = tid >> 5;
+
+    if (tid == 0) {
+        mbar_init(smem_u32(&misc->bar_q), 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
+            mbar_init(smem_u32(&misc->bar_vfull[b]), 1);
+            mbar_init(smem_u32(&misc->bar_kvempty[b]), 1);
+            mbar_init(smem_u32(&misc->bar_sfull[b]), 1);
+            mbar_init(smem_u32(&misc->bar_pfull[b]), 128);
+            mbar_init(smem_u32(&misc->bar_odone[b]), 1);
+        }
+        misc->abort = 0;
+        misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
+        fence_mbar_init();
+        if (P.has_prefill) {
+            tma_prefetch_desc(&P.tm_q);
+            tma_prefetch_desc(&P.tm_k);
+            tma_prefetch_desc(&P.tm_v);
+            tma_prefetch_desc(&P.tm_kpool);
+            tma_prefetch_desc(&P.tm_vpool);
+        }
+    }
+    if (P.has_prefill && warp == 1) {
+        tmem_alloc(smem_u32(&misc->tmem_base), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = P.has_prefill ? misc->tmem_base : 0u;
+
+    uint32_t tile_cnt = 0, item_no = 0;
+    int buf = 0;
+    for (;;) {
+        const int idx = misc->item_idx[buf];
+        if (idx >= P.n_items || misc->abort)
+            break;
+        if (tid == 0)
+            misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
+        const int4 it = P.items[idx];
+        if (it.x == ITEM_PREFILL) {
+            prefill_item(P, smem, misc, tmem, it.y, it.z,
+                         tile_cnt, item_no);
+            const int nA = (P.chunk_start + kTileN - 1) / kTileN;
+            tile_cnt += nA + it.y + 1;
+            item_no += 1;
+        } else {
+            decode_item(P, smem, misc, it.y, it.z, it.w);
+        }
+        fence_proxy_async_smem();  // generic smem accesses before later TMA writes
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        buf ^= 1;
+    }
+
+    if (misc->abort) {
+        // give in-flight copies and MMAs time to land before TMEM is freed
+        const uint64_t t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 200000ull)
+            __nanosleep(1000);
+        __syncthreads();
+    }
+    if (P.has_prefill && warp == 1)
+        tmem_dealloc(tmem, kTmemCols);
+    if (tid == 0) {
+        __threadfence();
+        const uint32_t prev = atomicAdd(P.work_cnt + 1, 1u);
+        if (prev == gridDim.x - 1) {
+            P.work_cnt[0] = 0u;
+            P.work_cnt[1] = 0u;
+            __threadfence();
+        }
+    }
+}
+
+// Standalone KV append: one warp per (token, KV head), 16-byte vectors.
+__global__ void kv_append_kernel(const int32_t *__restrict__ slots, int n_tokens, int hkv,
+                                 int num_pages, const uint16_t *__restrict__ k,
+                                 const uint16_t *__restrict__ v, uint16_t *k_pool,
+                                 uint16_t *v_pool, uint32_t *err)
+{
+    const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (gw >= n_tokens * hkv)
+        return;
+    const int tok = gw / hkv, h = gw % hkv;
+    const int slot = __ldg(slots + tok);
+    if (slot < 0)
+        return;
+    if (slot >= num_pages * kPage) {
+        if (lane == 0)
+            atomicOr(err, ERR_SLOT);
+        return;
+    }
+    const size_t dst = (((size_t)(slot / kPage) * hkv + h) * kPage + slot % kPage) * kHeadDim;
+    const size_t src = ((size_t)tok * hkv + h) * kHeadDim;
+    const int c = lane & 15;
+    if (lane < 16)
+        reinterpret_cast<uint4 *>(k_pool + dst)[c] = __ldg(reinterpret_cast<const uint4 *>(k + src) + c);
+    else
+        reinterpret_cast<uint4 *>(v_pool + dst)[c] = __ldg(reinterpret_cast<const uint4 *>(v + src) + c);
+}
+
+// ---------------------------------------------------------------------------
+// Host-side launchers (called from mx_api.cpp)
+cudaError_t init_layer_kernel()
+{
+    return cudaFuncSetAttribute(mixed_layer_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kSmemTotal);
+}
+
+cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream)
+{
+    mixed_layer_kernel<<<grid, kThreads, kSmemTotal, stream>>>(P);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int num_pages,
+                             const uint16_t *k, const uint16_t *v, uint16_t *k_pool,
+                             uint16_t *v_pool, uint32_t *err, cudaStream_t stream)
+{
+    const long long warps = (long long)n_tokens * hkv;
+    const int block = 256;
+    const long long grid = (warps * 32 + block - 1) / block;
+    if (grid == 0)
+        return cudaSuccess;
+    kv_append_kernel<<<(unsigned)grid, block, 0, stream>>>(slots, n_tokens, hkv, num_pages, k, v,
+                                                          k_pool, v_pool, err);
+    return cudaGetLastError();
+}
+
+}  // namespace mx

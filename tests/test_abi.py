@@ -1,0 +1,62 @@
+"""The C-ABI library loads and exports every entry point include/*.h
+declares; argument checks that need no GPU return their error codes."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_38386_gb300 import build as b
+    if not os.path.exists(b.LIB):
+        b.build_library()
+    from paper_2609_38386_gb300 import _binding
+    return _binding.load()
+
+
+def _declared():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        names.update(re.findall(r"^int\s+(mx_\w+)\s*\(", open(h).read(), re.M))
+    return names
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for must in ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",
+                 "mx_iteration"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    from paper_2609_38386_gb300 import _binding
+    for name in _declared():
+        assert hasattr(lib, name), name
+    assert set(_binding.EXPORTS) >= _declared()
+
+
+def test_null_and_geometry_checks_without_gpu(lib):
+    from paper_2609_38386_gb300._binding import mx_geom
+    assert lib.mx_destroy(None) == 0
+    assert lib.mx_mixed_attention(None, None, None, None) == -1
+    assert lib.mx_iteration(None, None, 0, None, None, None) == -1
+    assert lib.mx_error_detail(None, None, 0) == -1
+    assert lib.mx_set_option(None, 1, 0) == -1
+    h = ctypes.c_void_p()
+    bad = mx_geom(16, 8, 64, 16, 10, 1, 4, 8, 1)          # head_dim 64 unsupported
+    assert lib.mx_create(ctypes.byref(h), ctypes.byref(bad), 0) == -1
+    bad = mx_geom(24, 8, 128, 16, 10, 1, 4, 8, 1)         # n_rep 3 unsupported
+    assert lib.mx_create(ctypes.byref(h), ctypes.byref(bad), 0) == -1
+    try:
+        import torch
+        has_gpu = torch.cuda.is_available()
+    except Exception:
+        has_gpu = False
+    if not has_gpu:
+        good = mx_geom(16, 8, 128, 16, 10, 1, 4, 8, 1)
+        assert lib.mx_create(ctypes.byref(h), ctypes.byref(good), 0) == -6   # MX_EDEVICE

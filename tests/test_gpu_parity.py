@@ -1,0 +1,211 @@
+"""GPU parity: the CUDA path (through the C ABI) against the float64 oracle.
+
+Tolerance for attention outputs (bf16 vs float64): max abs <= 1e-2, mean abs
+<= 1e-3.  KV pages: bit-exact.  Sizes span several tiles, ragged tails,
+multi-split decodes and the degenerate cases (ctx = 0, p = 1, no decodes,
+no prefill).
+"""
+import numpy as np
+import pytest
+
+from tests import harness
+from tests.harness import MAX_ABS, MEAN_ABS, Case
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+def _ok(err):
+    assert err["finite"], "non-finite outputs"
+    assert err["max_abs"] <= MAX_ABS, err
+    assert err["mean_abs"] <= MEAN_ABS, err
+    assert err["pools_exact"], "KV pages differ from the oracle"
+
+
+def test_small_config_full_parity():
+    case = harness.config_case("qwen3-0.6b-attn-1layer-small")
+    res = case.run_gpu()
+    _ok(case.check(res))
+
+
+@pytest.mark.parametrize("ctx", [[0], [1, 15, 16, 17], [5, 300, 1023, 1024, 2049],
+                                 [4095, 4096, 7000]])
+@pytest.mark.parametrize("hq", [16, 64])
+def test_decode_only(ctx, hq):
+    case = Case(hq, ctx, seed=len(ctx) + hq)
+    res = case.run_gpu()
+    _ok(case.check(res))
+
+
+@pytest.mark.parametrize("hq", [8, 16, 32, 64])
+def test_decode_n_rep(hq):
+    case = Case(hq, [33, 700, 129], seed=hq)
+    _ok(case.check(case.run_gpu()))
+
+
+@pytest.mark.parametrize("split", [128, 256, 4096])
+def test_decode_split_sizes(split):
+    from paper_2609_38386_gb300 import MX_OPT_SPLIT_KEYS
+    case = Case(32, [3000, 129, 128, 4500], seed=split)
+    res = case.run_gpu(options={MX_OPT_SPLIT_KEYS: split})
+    assert res["plan"]["split_keys"] == split
+    _ok(case.check(res))
+
+
+@pytest.mark.parametrize("cs,p", [(0, 1), (0, 7), (0, 128), (0, 129), (5, 60), (128, 128),
+                                  (200, 300), (1000, 384), (16, 255)])
+def test_prefill_only(cs, p):
+    case = Case(16, [], chunk_start=cs, p_t=p, prompt_len=cs + p + 9, seed=cs + p)
+    _ok(case.check(case.run_gpu()))
+
+
+@pytest.mark.parametrize("hq", [8, 32, 64])
+def test_prefill_n_rep(hq):
+    case = Case(hq, [], chunk_start=130, p_t=200, seed=hq)
+    _ok(case.check(case.run_gpu()))
+
+
+@pytest.mark.parametrize("hq,ctx,cs,p", [(16, [64, 256, 100, 200], 128, 128),
+                                         (32, [0, 17, 1500, 3333, 64], 77, 257),
+                                         (64, [2000, 9], 512, 640)])
+def test_mixed(hq, ctx, cs, p):
+    case = Case(hq, ctx, chunk_start=cs, p_t=p, seed=hq + p)
+    _ok(case.check(case.run_gpu()))
+
+
+def test_paging_invariance_bit_identical():
+    a = Case(16, [100, 37, 900], chunk_start=50, p_t=150, seed=3)
+    b = Case(16, [100, 37, 900], chunk_start=50, p_t=150, seed=3)
+    # b: same logical contents, different physical pages
+    from synth import workload as wl
+    lay_b = wl.make_layout(b.geom, b.layout.capacities, seed=999, spare_pages=5)
+    ka, va = a.pools0()
+    perm_a = a.layout.page_table
+    kb = np.zeros(lay_b.pool_shape(), np.uint16)
+    vb = np.zeros(lay_b.pool_shape(), np.uint16)
+    for s in range(perm_a.shape[0]):
+        for lp in range(perm_a.shape[1]):
+            if perm_a[s, lp] >= 0:
+                kb[lay_b.page_table[s, lp]] = ka[perm_a[s, lp]]
+                vb[lay_b.page_table[s, lp]] = va[perm_a[s, lp]]
+    b.layout = lay_b
+    b.slots = b.it.slots(lay_b)
+    b._k_pool0, b._v_pool0 = kb, vb
+    ra, rb = a.run_gpu(), b.run_gpu()
+    np.testing.assert_array_equal(ra["out"], rb["out"])
+
+
+def test_run_to_run_deterministic():
+    case = Case(32, [1200, 50, 4000], chunk_start=300, p_t=260, seed=5)
+    r1, r2 = case.run_gpu(), case.run_gpu()
+    np.testing.assert_array_equal(r1["out"], r2["out"])
+    np.testing.assert_array_equal(r1["k_pool"], r2["k_pool"])
+
+
+def test_chunked_equals_unchunked_within_tolerance():
+    """Prefilling a prompt in chunks gives the one-shot outputs (the paper's
+    exact-output agreement, §5.1), here within the bf16 tolerance."""
+    L = 640
+    base = Case(16, [], chunk_start=0, p_t=L, seed=11)
+    full = base.run_gpu()["out"]
+    from paper_2609_38386_gb300 import Context  # noqa: F401
+    outs = []
+    k0, v0 = base.pools0()
+    kp = torch.from_numpy(k0.view(np.int16)).cuda()
+    vp = torch.from_numpy(v0.view(np.int16)).cuda()
+    ctx = base.make_context()
+    pt = torch.from_numpy(base.layout.page_table).cuda()
+    for cs in range(0, L, 192):
+        p = min(192, L - cs)
+        sl = torch.from_numpy(base.slots[cs:cs + p].copy()).cuda()
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a[cs:cs + p]).view(np.int16)).cuda()
+        q, k, v = t(base.q), t(base.k), t(base.v)
+        out = torch.empty((p, 16, 128), dtype=torch.int16, device="cuda")
+        desc = ctx.make_desc(decode_seq_ids=[], decode_ctx_lens=[], prefill_seq_id=0,
+                             chunk_start=cs, p_t=p, page_table=pt, slots=sl)
+        ctx.mixed_attention(desc, ctx.make_bufs(q, k, v, kp, vp, out))
+        ctx.sync_status()
+        outs.append(out.cpu().numpy().view(np.uint16))
+    ctx.close()
+    chunked = np.concatenate(outs)
+    diff = np.abs(harness._bf16_to_f64(chunked) - harness._bf16_to_f64(full))
+    assert diff.max() <= MAX_ABS and diff.mean() <= MEAN_ABS
+
+
+def test_kv_append_standalone_bit_exact():
+    from paper_2609_38386_gb300 import Context
+    rng = np.random.default_rng(0)
+    num_pages, n = 40, 37
+    ctx = Context(num_q_heads=16, num_pages=num_pages, num_seqs=1, max_pages_per_seq=num_pages,
+                  max_tokens=64, max_decodes=1)
+    kp = torch.full((num_pages, 8, 16, 128), 0x1234, dtype=torch.int16, device="cuda")
+    vp = torch.full((num_pages, 8, 16, 128), 0x4321, dtype=torch.int16, device="cuda")
+    slots = rng.choice(num_pages * 16, size=n, replace=False).astype(np.int32)
+    slots[[3, 9]] = -1
+    k = torch.randint(-30000, 30000, (n, 8, 128), dtype=torch.int16, device="cuda")
+    v = torch.randint(-30000, 30000, (n, 8, 128), dtype=torch.int16, device="cuda")
+    ctx.kv_append(torch.from_numpy(slots).cuda(), k, v, kp, vp)
+    ctx.sync_status()
+    want_k = np.full((num_pages, 8, 16, 128), 0x1234, np.int16)
+    want_v = np.full((num_pages, 8, 16, 128), 0x4321, np.int16)
+    kh, vh = k.cpu().numpy(), v.cpu().numpy()
+    for t, s in enumerate(slots):
+        if s >= 0:
+            want_k[s // 16, :, s % 16] = kh[t]
+            want_v[s // 16, :, s % 16] = vh[t]
+    np.testing.assert_array_equal(kp.cpu().numpy(), want_k)
+    np.testing.assert_array_equal(vp.cpu().numpy(), want_v)
+    ctx.close()
+
+
+def test_bad_page_id_reported_not_trapped():
+    from paper_2609_38386_gb300 import MxError
+    case = Case(16, [40, 70], seed=1)
+    case.layout.page_table = case.layout.page_table.copy()
+    case.layout.page_table[1, 1] = case.layout.num_pages + 5   # outside the pool
+    with pytest.raises(MxError) as ei:
+        case.run_gpu()
+    assert "ERANGE_PAGE" in str(ei.value)
+    # the context and device stay usable
+    ok = Case(16, [40, 70], seed=1)
+    _ok(ok.check(ok.run_gpu()))
+
+
+def test_host_validation_rejects_before_launch():
+    from paper_2609_38386_gb300 import MxError
+    case = Case(16, [40], chunk_start=10, p_t=20, seed=2)
+    ctx = case.make_context()
+    d = case.device_inputs()
+    bufs = ctx.make_bufs(d["q"], d["k"], d["v"], d["k_pool"], d["v_pool"], d["out"])
+    bad = ctx.make_desc(decode_seq_ids=[0], decode_ctx_lens=[10**6], prefill_seq_id=1,
+                        chunk_start=10, p_t=20, page_table=d["page_table"], slots=d["slots"])
+    with pytest.raises(MxError) as ei:
+        ctx.mixed_attention(bad, bufs)
+    assert "ECAPACITY" in str(ei.value)
+    bad2 = ctx.make_desc(decode_seq_ids=[7], decode_ctx_lens=[10], prefill_seq_id=1,
+                         chunk_start=10, p_t=20, page_table=d["page_table"], slots=d["slots"])
+    with pytest.raises(MxError):
+        ctx.mixed_attention(bad2, bufs)
+    ctx.close()
+
+
+def test_iteration_returns_device_time():
+    case = Case(16, [300, 500, 1000], chunk_start=256, p_t=256, seed=4)
+    ctx = case.make_context()
+    layers = []
+    devs = []
+    for _ in range(3):
+        d = case.device_inputs()
+        devs.append(d)
+        layers.append(ctx.make_bufs(d["q"], d["k"], d["v"], d["k_pool"], d["v_pool"], d["out"]))
+    desc = case.desc(ctx, devs[0])
+    us = ctx.iteration(desc, layers)
+    assert 0.0 < us < 1e6
+    # each layer produced the one-layer result
+    ref = case.check({"out": devs[0]["out"].cpu().numpy().view(np.uint16),
+                      "k_pool": devs[0]["k_pool"].cpu().numpy().view(np.uint16),
+                      "v_pool": devs[0]["v_pool"].cpu().numpy().view(np.uint16)})
+    _ok(ref)
+    np.testing.assert_array_equal(devs[1]["out"].cpu().numpy(), devs[0]["out"].cpu().numpy())
+    ctx.close()
