@@ -1,0 +1,491 @@
+#!/usr/bin/env python
+"""Mixed-iteration benchmark on GB300: prints ONE JSON line.
+
+Workload (default): Qwen3-0.6B attention geometry (16 Q / 8 KV heads, head dim
+128, bf16, 16-token pages), 28 layer calls per iteration with distinct
+per-layer pools, 32 decodes with cached contexts uniform in [512, 4096], and
+one 8192-token prompt prefilled beside them with chunk size p swept over
+{0, 256, 512, 1024, 2048, 4096}, every chunk in order (63 iterations).  One
+step = that whole sweep.  Inputs are seeded synthetic N(0,1) bf16 values,
+resident in HBM before timing (per-layer pools of ~335 MB, far above L2).
+
+`value` = tokens (decode tokens + prompt tokens) per second of device time,
+from CUDA events on the launching stream; `e2e` = the same through the C-ABI
+iteration call with host buffers (q/k/v copied in, outputs copied out, every
+iteration synchronised on its completion time).  `--impl reference` times the
+float64 CPU oracle on a bounded sample instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = ("mixed-iteration device µs & tokens/s; % of HBM/tensor roofline per chunk size")
+UNIT = "tokens/s"
+DEFAULT_CONFIG = "qwen3-0.6b-attn-28L-chunk-sweep"
+KERNEL_SRC = os.path.join(ROOT, "paper_2609_38386_gb300", "csrc", "mx_layer.cu")
+TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "mixed_layer_qwen06b_sweep.md")
+
+
+# ----------------------------------------------------------------- helpers
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]),
+                "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def kernel_hash():
+    h = hashlib.sha256()
+    for f in (KERNEL_SRC, os.path.join(ROOT, "paper_2609_38386_gb300", "csrc", "mx_ptx.cuh"),
+              os.path.join(ROOT, "paper_2609_38386_gb300", "csrc", "mx_internal.h")):
+        h.update(open(f, "rb").read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic():
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    if not os.path.exists(TRAFFIC_SUMMARY):
+        return None
+    txt = open(TRAFFIC_SUMMARY).read()
+    m_h = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", txt)
+    m_t = re.search(r"dram_bytes_per_launch_full_workload:\s*([0-9.eE+]+)", txt)
+    if not m_h or not m_t or m_h.group(1) != kernel_hash():
+        return None
+    return float(m_t.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = os.path.join("/tmp", f"mx_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", self.gpu_id], stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, val in zip(self.NAMES, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        os.unlink(self.path)
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ------------------------------------------------------------ GPU workload
+class Workload:
+    """Device-resident inputs of every iteration of a sweep, per layer."""
+
+    def __init__(self, cfg, device, seed_offset=0, layers=None):
+        import torch
+
+        import synth
+        from paper_2609_38386_gb300 import Context
+        from synth import device as sdev
+        from synth import workload as wl
+
+        self.cfg = cfg
+        self.geom = g = cfg.geom
+        self.L = layers or cfg.n_layers
+        self.layout = lay = cfg.layout()
+        self.its = cfg.iterations()
+        self.seed = cfg.seed + seed_offset
+        self.max_tok = max(it.n_tokens for it in self.its)
+        self.ctx = Context(num_q_heads=g.hq, num_kv_heads=g.hkv, num_pages=lay.num_pages,
+                           num_seqs=lay.num_seqs, max_pages_per_seq=lay.max_pages,
+                           max_tokens=self.max_tok, max_decodes=max(cfg.n_decodes, 1),
+                           device=device.index or 0)
+        self.page_table = torch.from_numpy(lay.page_table).to(device)
+        self.pools = []
+        for l in range(self.L):
+            kp = torch.empty(lay.pool_shape(), dtype=torch.int16, device=device)
+            vp = torch.empty(lay.pool_shape(), dtype=torch.int16, device=device)
+            sdev.fill_(kp, wl.pool_base(self.seed, l, synth.STREAM_KPOOL))
+            sdev.fill_(vp, wl.pool_base(self.seed, l, synth.STREAM_VPOOL))
+            self.pools.append((kp, vp))
+        self.outs = [torch.empty((self.max_tok, g.hq, g.head_dim), dtype=torch.int16,
+                                 device=device) for _ in range(self.L)]
+        self.descs, self.layer_arrays, self.inputs, self.slots = [], [], [], []
+        for it in self.its:
+            sl = torch.from_numpy(it.slots(lay)).to(device)
+            self.slots.append(sl)
+            bufs, keep = [], []
+            for l in range(self.L):
+                q = torch.empty((it.n_tokens, g.hq, g.head_dim), dtype=torch.int16, device=device)
+                k = torch.empty((it.n_tokens, g.hkv, g.head_dim), dtype=torch.int16, device=device)
+                v = torch.empty_like(k)
+                sdev.fill_tokens_(q, self.seed, l, synth.STREAM_Q, it)
+                sdev.fill_tokens_(k, self.seed, l, synth.STREAM_K, it)
+                sdev.fill_tokens_(v, self.seed, l, synth.STREAM_V, it)
+                keep.append((q, k, v))
+                kp, vp = self.pools[l]
+                bufs.append(self.ctx.make_bufs(q, k, v, kp, vp, self.outs[l]))
+            self.inputs.append(keep)
+            self.layer_arrays.append(self.ctx.layer_array(bufs))
+            self.descs.append(self.ctx.make_desc(
+                decode_seq_ids=it.decode_seq_ids, decode_ctx_lens=it.decode_ctx_lens,
+                prefill_seq_id=it.prefill_seq, chunk_start=it.chunk_start, p_t=it.p_t,
+                page_table=self.page_table, slots=sl))
+        torch.cuda.synchronize(device)
+        self.work = [wl.algorithmic_work(g, it) for it in self.its]
+        self.tokens_per_step = sum(it.n_tokens for it in self.its)
+
+    def run_step(self, events=None):
+        """Enqueue every iteration of the sweep (no host waits)."""
+        for i in range(len(self.its)):
+            if events is not None:
+                events[i].record()
+            self.ctx.iteration(self.descs[i], self.layer_arrays[i], wait=False)
+        if events is not None:
+            events[len(self.its)].record()
+
+
+def e2e_measure(w, steps, device):
+    """Same sweep through the iteration call with host buffers: per iteration,
+    copy every layer's q/k/v from pinned host memory, run the iteration and
+    wait for its completion time, copy every layer's output back."""
+    import torch
+    g, L = w.geom, w.L
+    per_tok_in = (g.hq + 2 * g.hkv) * g.head_dim
+    per_tok_out = g.hq * g.head_dim
+    max_in = L * w.max_tok * per_tok_in
+    max_out = L * w.max_tok * per_tok_out
+    h_in = torch.empty(max_in, dtype=torch.int16, pin_memory=True)
+    h_out = torch.empty(max_out, dtype=torch.int16, pin_memory=True)
+    d_in = torch.empty(max_in, dtype=torch.int16, device=device)
+    d_out = torch.empty(max_out, dtype=torch.int16, device=device)
+    # host contents: the largest iteration's device inputs, packed per layer
+    big = max(range(len(w.its)), key=lambda i: w.its[i].n_tokens)
+    off = 0
+    for l in range(L):
+        for t in w.inputs[big][l]:
+            n = t.numel()
+            h_in[off:off + n].copy_(t.reshape(-1).cpu())
+            off += n
+    layer_arrays, in_bytes, out_bytes = [], [], []
+    for i, it in enumerate(w.its):
+        n = it.n_tokens
+        bufs, o_in, o_out = [], 0, 0
+        for l in range(L):
+            q = d_in[o_in:o_in + n * g.hq * g.head_dim]
+            o_in += q.numel()
+            k = d_in[o_in:o_in + n * g.hkv * g.head_dim]
+            o_in += k.numel()
+            v = d_in[o_in:o_in + n * g.hkv * g.head_dim]
+            o_in += v.numel()
+            out = d_out[o_out:o_out + n * per_tok_out]
+            o_out += out.numel()
+            kp, vp = w.pools[l]
+            bufs.append(w.ctx.make_bufs(q, k, v, kp, vp, out))
+        layer_arrays.append(w.ctx.layer_array(bufs))
+        in_bytes.append(o_in * 2)
+        out_bytes.append(o_out * 2)
+    stream = torch.cuda.current_stream(device)
+
+    def one_step():
+        dev_us = []
+        for i in range(len(w.its)):
+            ni, no = in_bytes[i] // 2, out_bytes[i] // 2
+            d_in[:ni].copy_(h_in[:ni], non_blocking=True)
+            dev_us.append(w.ctx.iteration(w.descs[i], layer_arrays[i], stream=stream, wait=True))
+            h_out[:no].copy_(d_out[:no], non_blocking=True)
+            stream.synchronize()
+        return dev_us
+
+    one_step()  # warm-up
+    torch.cuda.synchronize(device)
+    t0 = time.perf_counter()
+    all_us = []
+    for _ in range(steps):
+        all_us += one_step()
+    torch.cuda.synchronize(device)
+    dt = time.perf_counter() - t0
+    return {"value": w.tokens_per_step * steps / dt, "unit": UNIT,
+            "h2d_bytes_per_step": int(sum(in_bytes)), "d2h_bytes_per_step": int(sum(out_bytes)),
+            "seconds": dt, "iteration_device_us_median": float(np.median(all_us))}
+
+
+# ------------------------------------------------------------- CPU oracle
+def oracle_sample(cfg, which="heavy"):
+    """A bounded slice of the workload for the CPU oracle: one layer call of
+    one iteration (heavy: the p=2048 chunk at 6144; light: the p=256 chunk at
+    4096).  Returns (fn, tokens_per_iteration_equivalent, description)."""
+    import oracle
+    import synth
+    from synth import workload as wl
+    its = cfg.iterations()
+    want = (2048, 6144) if which == "heavy" else (256, 4096)
+    it = next((x for x in its if (x.chunk_size, x.chunk_start) == want), its[-1])
+    lay = cfg.layout()
+    g = cfg.geom
+    q = wl.host_tokens(cfg.seed, 0, synth.STREAM_Q, it, g.hq)
+    k = wl.host_tokens(cfg.seed, 0, synth.STREAM_K, it, g.hkv)
+    v = wl.host_tokens(cfg.seed, 0, synth.STREAM_V, it, g.hkv)
+    # compact pool: the pages this iteration reads or writes
+    ps = g.page_size
+    seqs = list(it.decode_seq_ids) + ([it.prefill_seq] if it.p_t else [])
+    nkeys = list(it.decode_ctx_lens + 1) + ([it.chunk_start + it.p_t] if it.p_t else [])
+    pages = np.unique(np.concatenate([lay.page_table[s, :-(-int(n) // ps)]
+                                      for s, n in zip(seqs, nkeys)]))
+    remap = np.full(lay.num_pages, -1, np.int64)
+    remap[pages] = np.arange(len(pages))
+    pe = g.hkv * ps * g.head_dim
+    shp = (len(pages), g.hkv, ps, g.head_dim)
+    kp0 = synth.values_pages(wl.pool_base(cfg.seed, 0, synth.STREAM_KPOOL), pages, pe).reshape(shp)
+    vp0 = synth.values_pages(wl.pool_base(cfg.seed, 0, synth.STREAM_VPOOL), pages, pe).reshape(shp)
+    pt = np.where(lay.page_table >= 0, remap[np.maximum(lay.page_table, 0)], -1).astype(np.int32)
+    sl = it.slots(lay).astype(np.int64)
+    sl = (remap[sl // ps] * ps + sl % ps).astype(np.int32)
+
+    def fn():
+        kp, vp = kp0.copy(), vp0.copy()
+        oracle.mixed_attention(q=q, k=k, v=v, k_pool=kp, v_pool=vp, page_table=pt, slots=sl,
+                               decode_seq_ids=it.decode_seq_ids,
+                               decode_ctx_lens=it.decode_ctx_lens, prefill_seq=it.prefill_seq,
+                               chunk_start=it.chunk_start, p_t=it.p_t)
+
+    desc = (f"one layer call of the p={it.p_t} iteration at chunk_start={it.chunk_start} "
+            f"({it.n_decodes} decodes + {it.p_t} chunk rows, all {g.hq} heads); tokens/s "
+            f"scaled to the {cfg.n_layers}-layer iteration")
+    return fn, it.n_tokens, desc
+
+
+def cpu_baseline(cfg, which="heavy"):
+    import oracle
+    fn, ntok, desc = oracle_sample(cfg, which)
+    t0 = time.perf_counter()
+    fn()
+    dt = time.perf_counter() - t0
+    return {"value": ntok / (dt * cfg.n_layers), "unit": UNIT, "cores": oracle.max_threads(),
+            "kind": "oracle", "sample": desc, "seconds": dt}
+
+
+# ------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--profile", action="store_true",
+                    help="small case for ncu: 2 layers, iterations of --profile-chunk only")
+    ap.add_argument("--profile-chunk", type=int, default=2048)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+
+    ws, rank, local = dist_setup()
+    from synth import workload as wl
+    cfg = wl.CONFIGS[args.config]
+    config = {"workload": cfg.name, "q_heads": cfg.hq, "kv_heads": 8, "head_dim": 128,
+              "page_size": 16, "layers": cfg.n_layers, "decodes": cfg.n_decodes,
+              "decode_ctx": f"{cfg.ctx_dist}[{cfg.ctx_lo},{cfg.ctx_hi}]",
+              "prompt_len": cfg.prompt_len, "chunk_sizes": list(cfg.chunk_sizes),
+              "iterations_per_step": len(cfg.iterations()),
+              "l2": "inputs larger than L2: each iteration reads 28 distinct ~335 MB "
+                    "per-layer pools", "parallelism": f"replicas{ws}"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        import oracle
+        fn, ntok, desc = oracle_sample(cfg, "light")
+        for _ in range(args.warmup):
+            fn()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            fn()
+        dt = time.perf_counter() - t0
+        val = ntok * args.steps / (dt * cfg.n_layers)
+        line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT,
+                "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": config,
+                "cpu_baseline": {"value": val, "unit": UNIT, "cores": oracle.max_threads(),
+                                 "kind": "oracle", "sample": desc},
+                "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    import torch
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    peaks = load_peaks()
+
+    layers = 2 if args.profile else None
+    w = Workload(cfg, device, seed_offset=rank, layers=layers)
+    if args.profile:
+        keep = [i for i, it in enumerate(w.its) if it.chunk_size == args.profile_chunk][-2:]
+        w.its = [w.its[i] for i in keep]
+        w.descs = [w.descs[i] for i in keep]
+        w.layer_arrays = [w.layer_arrays[i] for i in keep]
+        w.work = [w.work[i] for i in keep]
+        w.tokens_per_step = sum(it.n_tokens for it in w.its)
+        config["workload"] += f"-profile-{w.L}L-p{args.profile_chunk}"
+
+    def barrier():
+        if ws > 1:
+            torch.distributed.barrier()
+
+    for _ in range(max(args.warmup, 0)):
+        w.run_step()
+    w.ctx.sync_status()
+    torch.cuda.synchronize(device)
+
+    n_it = len(w.its)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_it + 1)]
+           for _ in range(args.steps)]
+    gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
+    sampler = ClockSampler(gpu_id)
+    barrier()
+    torch.cuda.synchronize(device)
+    sampler.start()
+    time.sleep(0.25)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record()
+    for s in range(args.steps):
+        w.run_step(evs[s])
+    t_end.record()
+    torch.cuda.synchronize(device)
+    clocks = sampler.stop()
+    barrier()
+    w.ctx.sync_status()
+    total_ms = t_start.elapsed_time(t_end)
+    if ws > 1:
+        t = torch.tensor([total_ms], device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    it_us = np.array([[evs[s][i].elapsed_time(evs[s][i + 1]) * 1e3 for i in range(n_it)]
+                      for s in range(args.steps)])          # [steps][iterations]
+    L = w.L
+    hbm = peaks["hbm_gbs"] * 1e9
+    tfl = peaks["bf16_tflops_sustained"] * 1e12
+    B = np.array([L * b for b, _ in w.work], dtype=np.float64)
+    F = np.array([L * f for _, f in w.work], dtype=np.float64)
+    t_it = it_us.mean(axis=0) * 1e-6                         # seconds per iteration
+    per_chunk = {}
+    p0_p99 = None
+    for p in sorted(set(it.chunk_size for it in w.its)):
+        idx = [i for i, it in enumerate(w.its) if it.chunk_size == p]
+        samples = it_us[:, idx].ravel()
+        toks = sum(w.its[i].n_tokens for i in idx)
+        t_sum = t_it[idx].sum()
+        roof = sum(max(F[i] / tfl, B[i] / hbm) for i in idx)
+        p99 = float(np.percentile(samples, 99))
+        if p == 0:
+            p0_p99 = p99
+        per_chunk[str(p)] = {
+            "iterations": len(idx), "samples": int(samples.size),
+            "device_us_p50": float(np.percentile(samples, 50)), "device_us_p99": p99,
+            "tokens_per_s": toks / t_sum,
+            "roofline_us_per_iter": roof / len(idx) * 1e6,
+            "roofline_frac": roof / t_sum,
+            "bound": "tensor" if sum(F[idx]) / tfl > sum(B[idx]) / hbm else "hbm",
+            "hbm_gbs": float(B[idx].sum() / t_sum / 1e9),
+            "tflops": float(F[idx].sum() / t_sum / 1e12)}
+    if p0_p99:
+        for v in per_chunk.values():
+            v["p99_vs_decode_only"] = v["device_us_p99"] / p0_p99
+
+    t_total = t_it.sum()
+    bound = "tensor" if F.sum() / tfl > B.sum() / hbm else "hbm"
+    if bound == "hbm":
+        achieved, peak, unit = B.sum() / t_total / 1e9, peaks["hbm_gbs"], "GB/s"
+    else:
+        achieved, peak, unit = F.sum() / t_total / 1e12, peaks["bf16_tflops_sustained"], "TFLOP/s"
+    traffic = committed_traffic()
+    roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+                "frac": achieved / peak, "traffic": traffic,
+                "algorithmic_bytes_per_launch": float(B.sum() / (L * n_it)),
+                "algorithmic_flops_per_launch": float(F.sum() / (L * n_it)),
+                "avg_launch_us": float(t_total / (L * n_it) * 1e6),
+                "max_bound_frac": float(sum(max(F[i] / tfl, B[i] / hbm) for i in range(n_it))
+                                        / t_total),
+                "peak_source": peaks["source"], "kernel": "mixed_layer_kernel"}
+
+    value = w.tokens_per_step * args.steps * ws / (total_ms * 1e-3)
+    plan = w.ctx.last_plan()
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded N(0,1) bf16, random page permutation)",
+            "config": config, "roofline": roofline, "per_chunk": per_chunk,
+            "gpu_launches": L * n_it * args.steps, "clocks": clocks,
+            "plan_last": plan}
+    if not args.no_e2e and not args.profile:
+        line["e2e"] = e2e_measure(w, max(1, min(args.steps, 3)), device)
+    if rank == 0 and ws == 1 and not args.no_cpu and not args.profile:
+        line["cpu_baseline"] = cpu_baseline(cfg)
+    if rank == 0:
+        print(json.dumps(line))
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -141,12 +141,14 @@ int mx_mixed_attention(mx_ctx *ctx, const mx_iter_desc *desc,
                        const mx_layer_bufs *bufs, void *stream);
 
 /* A whole iteration: the same schedule `desc` run through n_layers layers
- * (layers[l] holds layer l's tensors), one launch per layer.  Records CUDA
- * events before the first and after the last launch, waits for the second,
- * and stores the elapsed device time in microseconds in *device_us_out (the
- * L_t of Eq. 1 as completed on the device).  Reads and clears the device
- * error word: MX_ERANGE_PAGE / MX_ERANGE_SLOT / MX_ETIMEOUT if a kernel
- * flagged one (the time is still stored). */
+ * (layers[l] holds layer l's tensors), one launch per layer, planned once.
+ * With device_us_out != NULL: records CUDA events before the first and after
+ * the last launch, waits for the second, and stores the elapsed device time in
+ * microseconds in *device_us_out (the L_t of Eq. 1 as completed on the
+ * device); then reads and clears the device error word and returns
+ * MX_ERANGE_PAGE / MX_ERANGE_SLOT / MX_ETIMEOUT if a kernel flagged one (the
+ * time is still stored).  With device_us_out == NULL: only enqueues the
+ * launches on `stream` and returns (errors via mx_sync_status). */
 int mx_iteration(mx_ctx *ctx, const mx_iter_desc *desc, int32_t n_layers,
                  const mx_layer_bufs *layers, float *device_us_out,
                  void *stream);

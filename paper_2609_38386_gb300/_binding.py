@@ -170,13 +170,20 @@ class Context:
         self._check(self._lib.mx_mixed_attention(self._h, ctypes.byref(desc),
                                                  ctypes.byref(bufs), _stream_handle(stream)))
 
-    def iteration(self, desc, layers, stream=None):
-        """Run all layers; returns the device-completion time in microseconds."""
-        arr = (mx_layer_bufs * max(len(layers), 1))(*layers)
+    @staticmethod
+    def layer_array(layers):
+        """Pack a list of mx_layer_bufs into a C array (reusable across calls)."""
+        return (mx_layer_bufs * max(len(layers), 1))(*layers), len(layers)
+
+    def iteration(self, desc, layers, stream=None, wait=True):
+        """Run all layers.  wait=True: returns the device-completion time in
+        microseconds (CUDA events, synchronised).  wait=False: enqueue only."""
+        arr, n = layers if isinstance(layers, tuple) else self.layer_array(layers)
         us = ctypes.c_float()
-        self._check(self._lib.mx_iteration(self._h, ctypes.byref(desc), len(layers), arr,
-                                           ctypes.byref(us), _stream_handle(stream)))
-        return float(us.value)
+        self._check(self._lib.mx_iteration(self._h, ctypes.byref(desc), n, arr,
+                                           ctypes.byref(us) if wait else None,
+                                           _stream_handle(stream)))
+        return float(us.value) if wait else None
 
     def sync_status(self, stream=None):
         self._check(self._lib.mx_sync_status(self._h, _stream_handle(stream)))

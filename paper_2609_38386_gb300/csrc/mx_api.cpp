@@ -545,8 +545,9 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     int rc = validate(c, d);
     if (rc)
         return rc;
-    if (n_layers < 0 || (n_layers > 0 && !layers) || !device_us_out)
-        return fail(c, MX_EINVAL, "bad n_layers / layers / device_us_out");
+    if (n_layers < 0 || (n_layers > 0 && !layers))
+        return fail(c, MX_EINVAL, "bad n_layers / layers");
+    const bool timed = device_us_out != nullptr;
     const int n_tok = d->n_decodes + d->p_t;
     for (int l = 0; l < n_layers; ++l)
         if ((rc = validate_bufs(c, layers + l, n_tok)))
@@ -562,14 +563,16 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     for (int l = 0; work && l < n_layers; ++l)
         if ((rc = make_params(c, d, layers + l, pl, &params[l])))
             return rc;
-    cudaError_t e = cudaEventRecord(c->ev_start, st);
-    if (e != cudaSuccess)
+    cudaError_t e;
+    if (timed && (e = cudaEventRecord(c->ev_start, st)) != cudaSuccess)
         return cuda_fail(c, e, "cudaEventRecord(start)");
     for (int l = 0; work && l < n_layers; ++l) {
         e = launch_mixed_layer(params[l], grid_for(c, pl), st);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "mixed_layer launch");
     }
+    if (!timed)
+        return MX_OK;
     if ((e = cudaEventRecord(c->ev_end, st)) != cudaSuccess)
         return cuda_fail(c, e, "cudaEventRecord(end)");
     if ((e = cudaEventSynchronize(c->ev_end)) != cudaSuccess)

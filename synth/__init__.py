@@ -20,6 +20,10 @@ host bit for bit without reading device memory.
 """
 from __future__ import annotations
 
+import ctypes
+import os
+import subprocess
+
 import numpy as np
 
 TABLE_BITS = 20
@@ -77,10 +81,57 @@ def values(base: int, idx, table: np.ndarray | None = None) -> np.ndarray:
     return t[(h >> np.uint64(64 - TABLE_BITS)).astype(np.int64)]
 
 
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_HOSTLIB = os.path.join(_HERE, "libsynth_host.so")
+_host = None
+
+
+def _hostgen():
+    """The C version of the same formula (OpenMP), built on first use."""
+    global _host
+    if _host is None:
+        src = os.path.join(_HERE, "hostgen.c")
+        if (not os.path.exists(_HOSTLIB)
+                or os.path.getmtime(_HOSTLIB) < os.path.getmtime(src)):
+            tmp = _HOSTLIB + f".tmp{os.getpid()}"
+            subprocess.check_call(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared",
+                                   "-o", tmp, src])
+            os.replace(tmp, _HOSTLIB)
+        lib = ctypes.CDLL(_HOSTLIB)
+        P, i64, u64 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_uint64
+        lib.synth_range.argtypes = [P, i64, u64, u64, P]
+        lib.synth_range.restype = None
+        lib.synth_pages.argtypes = [P, P, i64, i64, u64, P]
+        lib.synth_pages.restype = None
+        _host = lib
+    return _host
+
+
+def values_range(base: int, start: int, n: int, table: np.ndarray | None = None) -> np.ndarray:
+    """Elements [start, start + n) of a stream (C fast path)."""
+    t = normal_table() if table is None else table
+    out = np.empty(int(n), dtype=np.uint16)
+    if n:
+        _hostgen().synth_range(out.ctypes.data, int(n), ctypes.c_uint64(base),
+                               ctypes.c_uint64(int(start)), t.ctypes.data)
+    return out
+
+
+def values_pages(base: int, pages, page_elems: int, table: np.ndarray | None = None) -> np.ndarray:
+    """Elements of whole pages (page p covers [p*page_elems, (p+1)*page_elems))."""
+    t = normal_table() if table is None else table
+    pg = np.ascontiguousarray(np.asarray(pages, dtype=np.int64))
+    out = np.empty(len(pg) * int(page_elems), dtype=np.uint16)
+    if len(pg):
+        _hostgen().synth_pages(out.ctypes.data, pg.ctypes.data, len(pg), int(page_elems),
+                               ctypes.c_uint64(base), t.ctypes.data)
+    return out
+
+
 def fill(base: int, shape, table: np.ndarray | None = None) -> np.ndarray:
     """A whole tensor of the stream, element i at flat index i."""
     n = int(np.prod(shape))
-    return values(base, np.arange(n, dtype=np.uint64), table).reshape(shape)
+    return values_range(base, 0, n, table).reshape(shape)
 
 
 # Stream identifiers: one per (layer, tensor) so that layers are independent.

@@ -48,3 +48,13 @@ def fill_(tensor, base: int, start: int = 0, stream=None):
     if rc != 0:
         raise RuntimeError(f"synth_fill failed: cuda error {rc}")
     return tensor
+
+
+def fill_tokens_(tensor, seed, layer, kind, it, stream=None):
+    """Device fill of a per-token input with the layout of
+    ``synth.workload.token_parts`` (decode rows, then chunk rows)."""
+    from synth import workload as wl
+    w = tensor.shape[1] * tensor.shape[2]
+    for row0, n, base, start in wl.token_parts(seed, layer, kind, it):
+        fill_(tensor[row0:row0 + n], base, start * w, stream)
+    return tensor

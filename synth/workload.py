@@ -16,6 +16,8 @@ import math
 
 import numpy as np
 
+import synth
+
 PAGE = 16
 HKV = 8
 HEAD_DIM = 128
@@ -218,3 +220,34 @@ def algorithmic_work(geom: Geometry, it: IterSpec):
         B += s * kv_tok + 2 * p * kv_tok + p * qo_tok + 4 * (-(-(s + p) // geom.page_size))
         F += 4 * geom.hq * geom.head_dim * (p * s + p * (p + 1) // 2)
     return int(B), int(F)
+
+
+def token_parts(seed: int, layer: int, kind: int, it: IterSpec):
+    """Where the rows of a per-token input ([n_tokens][heads][128]) come from.
+
+    Returns (row0, n_rows, base, start_row) parts: decode rows come from the
+    iteration's own stream, chunk rows from the prompt's stream at the chunk's
+    positions, so a prompt's tokens have the same q/k/v however it is chunked.
+    """
+    parts = []
+    if it.n_decodes:
+        parts.append((0, it.n_decodes,
+                      synth.stream_base(seed, synth.stream_id(layer, kind, it.index + 1)), 0))
+    if it.p_t:
+        parts.append((it.n_decodes, it.p_t,
+                      synth.stream_base(seed, synth.stream_id(layer, kind, 0)), it.chunk_start))
+    return parts
+
+
+def host_tokens(seed: int, layer: int, kind: int, it: IterSpec, heads: int,
+                head_dim: int = HEAD_DIM) -> np.ndarray:
+    """Host copy of a per-token input, bit-identical to the device fill."""
+    w = heads * head_dim
+    out = np.empty((it.n_tokens, heads, head_dim), dtype=np.uint16)
+    for row0, n, base, start in token_parts(seed, layer, kind, it):
+        out[row0:row0 + n] = synth.values_range(base, start * w, n * w).reshape(n, heads, head_dim)
+    return out
+
+
+def pool_base(seed: int, layer: int, kind: int) -> int:
+    return synth.stream_base(seed, synth.stream_id(layer, kind, 0))

@@ -29,7 +29,7 @@ class Case:
     """One layer call: decodes (seq ids + cached lengths) and one chunk."""
 
     def __init__(self, hq, ctx_lens, chunk_start=0, p_t=0, prompt_len=None, seed=0,
-                 layer=0, salt=1, layout=None, spare_pages=1, device_pools=False):
+                 layer=0, salt=0, layout=None, spare_pages=1, device_pools=False):
         self.geom = wl.Geometry(hq)
         ctx = np.asarray(ctx_lens, dtype=np.int32)
         nd = len(ctx)
@@ -44,12 +44,7 @@ class Case:
         self.seed, self.layer, self.salt = seed, layer, salt
         self.device_pools = device_pools
         self.slots = self.it.slots(layout)
-        g = self.geom
-        n = self.n_tokens
-        self.q = synth.fill(self._base(synth.STREAM_Q), (n, g.hq, g.head_dim))
-        self.k = synth.fill(self._base(synth.STREAM_K), (n, g.hkv, g.head_dim))
-        self.v = synth.fill(self._base(synth.STREAM_V), (n, g.hkv, g.head_dim))
-        self._k_pool0 = self._v_pool0 = None
+        self._gen_tokens()
 
     @classmethod
     def from_config(cls, cfg: wl.SweepConfig, it_index: int, layer=0, device_pools=True):
@@ -58,22 +53,22 @@ class Case:
         c.geom = cfg.geom
         c.layout = cfg.layout()
         c.it = it
-        c.seed, c.layer, c.salt = cfg.seed, layer, it.index + 1
+        c.seed, c.layer, c.salt = cfg.seed, layer, 0
         c.device_pools = device_pools
         c.slots = it.slots(c.layout)
-        g, n = c.geom, it.n_tokens
-        c.q = synth.fill(c._base(synth.STREAM_Q), (n, g.hq, g.head_dim))
-        c.k = synth.fill(c._base(synth.STREAM_K), (n, g.hkv, g.head_dim))
-        c.v = synth.fill(c._base(synth.STREAM_V), (n, g.hkv, g.head_dim))
-        c._k_pool0 = c._v_pool0 = None
+        c._gen_tokens()
         return c
 
+    def _gen_tokens(self):
+        g, it = self.geom, self.it
+        self.q = wl.host_tokens(self.seed, self.layer, synth.STREAM_Q, it, g.hq)
+        self.k = wl.host_tokens(self.seed, self.layer, synth.STREAM_K, it, g.hkv)
+        self.v = wl.host_tokens(self.seed, self.layer, synth.STREAM_V, it, g.hkv)
+        self._k_pool0 = self._v_pool0 = None
+
     # ---------------------------------------------------------------- inputs
-    def _base(self, kind, salt=None):
-        s = self.salt if salt is None else salt
-        if kind in (synth.STREAM_KPOOL, synth.STREAM_VPOOL):
-            s = 0
-        return synth.stream_base(self.seed, synth.stream_id(self.layer, kind, s))
+    def _base(self, kind):
+        return wl.pool_base(self.seed, self.layer, kind)
 
     @property
     def n_tokens(self):
@@ -97,11 +92,9 @@ class Case:
     def pages0(self, pages):
         """Initial contents of the listed physical pages, regenerated on the host."""
         pe = self.page_elems()
-        pages = np.asarray(pages, dtype=np.uint64)
-        idx = (pages[:, None] * np.uint64(pe) + np.arange(pe, dtype=np.uint64)[None]).ravel()
         shp = (len(pages),) + self.pool_shape[1:]
-        kp = synth.values(self._base(synth.STREAM_KPOOL), idx).reshape(shp)
-        vp = synth.values(self._base(synth.STREAM_VPOOL), idx).reshape(shp)
+        kp = synth.values_pages(self._base(synth.STREAM_KPOOL), pages, pe).reshape(shp)
+        vp = synth.values_pages(self._base(synth.STREAM_VPOOL), pages, pe).reshape(shp)
         return kp, vp
 
     # ------------------------------------------------------------------ GPU

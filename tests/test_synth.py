@@ -59,3 +59,14 @@ def test_sweep_iterations_cover_every_chunk_in_order():
     lay = wl.SMALL.layout()
     sl = small[0].slots(lay)
     assert len(sl) == 4 + 128 and len(np.unique(sl)) == len(sl)
+
+
+def test_c_fast_path_matches_numpy_definition():
+    base = synth.stream_base(7, synth.stream_id(2, synth.STREAM_V, 3))
+    idx = np.arange(1000, 5000, dtype=np.uint64)
+    np.testing.assert_array_equal(synth.values_range(base, 1000, 4000), synth.values(base, idx))
+    pages = np.array([5, 0, 17], np.int64)
+    pe = 64
+    want = synth.values(base, (pages.astype(np.uint64)[:, None] * np.uint64(pe)
+                               + np.arange(pe, dtype=np.uint64)[None]).ravel())
+    np.testing.assert_array_equal(synth.values_pages(base, pages, pe), want)
