@@ -171,6 +171,35 @@ int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
                  int32_t *n_prefill_items);
 
+/* For callers that cannot allocate device memory (a host framework whose
+ * allocator owns the GPU, a plug-in with a fixed pre-reserved budget, a path
+ * that must not risk an allocation's implicit synchronisation or OOM).  The
+ * paper has no counterpart: this is a deployment variant of
+ * mx_mixed_attention that needs no context, because mx_create allocates.
+ *
+ * Same operation, layouts and descriptor as mx_mixed_attention (geom gives
+ * the geometry a context would hold; max_tokens / max_decodes are ignored).
+ * Its scratch (work list, split partials, counters, error word) is one fixed
+ * 4.24 MiB device array built into the library, which every GPU that loads
+ * the library holds until the process exits.  Limits: n_decodes <= 256,
+ * at most 4096 work items (prefill tiles = ceil(p_t / 128) * Hq, plus decode
+ * splits), at most 1024 split partials, num_kv_heads <= 16; a request beyond
+ * them returns MX_ECAPACITY and enqueues nothing.
+ *
+ * The call allocates nothing (no cudaMalloc/cudaFree, no allocating library
+ * routine).  The first call on a device does a one-time set-up (it resolves
+ * the array's device address and the kernel attributes), so make that first
+ * call before any stream capture.  Each call zeroes the counters it needs,
+ * uploads its work list, launches, waits for `stream`, and reads the error
+ * word, so it returns MX_ERANGE_PAGE / MX_ERANGE_SLOT / MX_ETIMEOUT like
+ * mx_iteration.  All calls on a GPU share the one array: calls whose GPU work
+ * overlaps (other streams, other host threads) race and must be serialised
+ * by the caller.  On failure a message is written to err_buf (up to err_len
+ * bytes) when err_buf is not NULL. */
+int mx_mixed_attention_noalloc(const mx_geom *geom, const mx_iter_desc *desc,
+                               const mx_layer_bufs *bufs, void *stream,
+                               char *err_buf, int32_t err_len);
+
 #ifdef __cplusplus
 }
 #endif

@@ -24,7 +24,7 @@ MX_OPT_GRID = 2
 # Names every C-ABI build must export (the declarations of include/mixattn.h).
 EXPORTS = ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",
            "mx_iteration", "mx_sync_status", "mx_error_detail", "mx_set_option",
-           "mx_last_plan")
+           "mx_last_plan", "mx_mixed_attention_noalloc")
 
 
 class MxError(RuntimeError):
@@ -74,6 +74,8 @@ def load():
             "mx_error_detail": [P, ctypes.c_char_p, i32],
             "mx_set_option": [P, i32, i64],
             "mx_last_plan": [P, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)],
+            "mx_mixed_attention_noalloc": [ctypes.POINTER(mx_geom), ctypes.POINTER(mx_iter_desc),
+                                           ctypes.POINTER(mx_layer_bufs), P, ctypes.c_char_p, i32],
         }
         for name, args in sig.items():
             f = getattr(lib, name)
