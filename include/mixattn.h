@@ -161,9 +161,13 @@ int mx_sync_status(mx_ctx *ctx, void *stream);
 int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
 
 /* Tunables.  MX_OPT_SPLIT_KEYS: keys per decode split (multiple of 128,
- * 0 = automatic).  MX_OPT_GRID: persistent grid size (0 = number of SMs). */
+ * 0 = automatic).  MX_OPT_GRID: persistent grid size (0 = number of SMs).
+ * MX_OPT_PREFILL_PIECE_TILES: at most this many 128-key tiles per prefill
+ * work item; longer causal tiles are split into pieces merged by
+ * log-sum-exp (0 = automatic, 65535 = never split). */
 #define MX_OPT_SPLIT_KEYS 1
 #define MX_OPT_GRID 2
+#define MX_OPT_PREFILL_PIECE_TILES 3
 int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 
 /* Number of work items and decode split length chosen for the last planned

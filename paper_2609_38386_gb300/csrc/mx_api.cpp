@@ -32,7 +32,9 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 constexpr int kPlanSlots = 4;         // ring of work-list buffers
-constexpr int kPartSlots = 16384;     // split partials capacity
+constexpr int kPartSlots = 16384;     // decode split partials capacity
+constexpr int kPrePartSlots = 1024;   // prefill piece partials capacity (64 KiB each)
+constexpr int kMinPieceTiles = 32;    // smallest prefill piece, in 128-key tiles
 constexpr int kMaxSplitKeys = kWarps * 32 * kPage;  // 4096: one page id per lane
 constexpr uint64_t kTimeoutNs = 1000000000ull;      // 1 s bound on in-kernel waits
 
@@ -48,6 +50,9 @@ struct mx_ctx {
     float *part_o = nullptr;
     float *part_lse = nullptr;
     uint32_t *merge_cnt = nullptr;
+    float *pre_o = nullptr;
+    float *pre_lse = nullptr;
+    uint32_t *pre_cnt = nullptr;
     uint32_t *work_cnt = nullptr;
     uint32_t *err = nullptr;
     uint8_t *plan_dev[kPlanSlots] = {};
@@ -62,8 +67,9 @@ struct mx_ctx {
     // options
     int split_keys_opt = 0;
     int grid_opt = 0;
+    int piece_tiles_opt = 0;
     // last plan
-    int last_items = 0, last_split = 0, last_prefill_items = 0;
+    int last_items = 0, last_split = 0, last_prefill_items = 0, last_piece_tiles = 0;
     std::string last_error;
 };
 
@@ -203,11 +209,58 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     const size_t items_off = (size_t)nd * sizeof(DecodeInfo);
     int4 *items = reinterpret_cast<int4 *>(host + items_off);
 
+    // Prefill tiles, split along their key tiles into pieces of at most
+    // piece_tiles tiles so that long causal rows spread over several SMs.
     int n = 0;
     const int n_qt = (d->p_t + kTileM - 1) / kTileM;
-    for (int t = n_qt - 1; t >= 0; --t)
-        for (int h = 0; h < hq; ++h)
-            items[n++] = make_int4(ITEM_PREFILL, t, h, 0);
+    const int nA = (d->chunk_start + kTileN - 1) / kTileN;
+    int64_t pre_work = 0;
+    for (int t = 0; t < n_qt; ++t)
+        pre_work += (int64_t)(nA + t + 1) * hq;
+    // Splitting costs a partial write and a merge; it pays only when the
+    // chunk has too few tiles to occupy the GPU (short chunks deep into a
+    // long prompt), so tiles are split only then, into >= 32-tile pieces.
+    int piece = c->piece_tiles_opt;
+    if (piece <= 0) {
+        if ((int64_t)n_qt * hq * 2 >= c->num_sms)
+            piece = 65535;
+        else
+            piece = (int)std::max<int64_t>(kMinPieceTiles, (pre_work + c->num_sms - 1) / c->num_sms);
+    }
+    auto count_pre_parts = [&](int pc) {
+        int64_t parts = 0;
+        for (int t = 0; t < n_qt; ++t) {
+            const int ns = (nA + t + 1 + pc - 1) / pc;
+            if (ns > 1)
+                parts += (int64_t)ns * hq;
+        }
+        return parts;
+    };
+    while (count_pre_parts(piece) > kPrePartSlots)
+        piece *= 2;
+    struct PItem { int tiles; int4 code; };
+    std::vector<PItem> pitems;
+    pitems.reserve(64);
+    int pre_part = 0;
+    for (int t = n_qt - 1; t >= 0; --t) {
+        const int nT = nA + t + 1;
+        const int ns = (nT + piece - 1) / piece;
+        for (int h = 0; h < hq; ++h) {
+            const int base = ns > 1 ? pre_part : 0;
+            if (ns > 1)
+                pre_part += ns;
+            for (int s2 = 0; s2 < ns; ++s2) {
+                const int len = (int)((int64_t)(s2 + 1) * nT / ns - (int64_t)s2 * nT / ns);
+                pitems.push_back({len, prefill_item_code(t, h, s2, ns, base)});
+            }
+        }
+    }
+    std::stable_sort(pitems.begin(), pitems.end(),
+                     [](const PItem &a, const PItem &b) { return a.tiles > b.tiles; });
+    if ((int64_t)pitems.size() > c->max_items)
+        return fail(c, MX_ECAPACITY, "%zu prefill items exceed capacity %d", pitems.size(), c->max_items);
+    for (const PItem &x : pitems)
+        items[n++] = x.code;
     const int n_prefill = n;
 
     int part = 0;
@@ -233,7 +286,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     std::stable_sort(ditems.begin(), ditems.end(),
                      [](const DItem &a, const DItem &b) { return a.keys > b.keys; });
     for (const DItem &x : ditems)
-        items[n++] = make_int4(ITEM_DECODE, x.i, x.h, x.s);
+        items[n++] = decode_item_code(x.i, x.h, x.s);
 
     const size_t bytes = items_off + (size_t)n * sizeof(int4);
     cudaError_t e = cudaMemcpyAsync(c->plan_dev[slot], host, bytes, cudaMemcpyHostToDevice, stream);
@@ -253,6 +306,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     c->last_items = n;
     c->last_split = split;
     c->last_prefill_items = n_prefill;
+    c->last_piece_tiles = piece;
     return MX_OK;
 }
 
@@ -288,6 +342,9 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->part_o = c->part_o;
     P->part_lse = c->part_lse;
     P->merge_cnt = c->merge_cnt;
+    P->pre_o = c->pre_o;
+    P->pre_lse = c->pre_lse;
+    P->pre_cnt = c->pre_cnt;
     P->work_cnt = c->work_cnt;
     P->err = c->err;
     P->n_items = pl.n_items;
@@ -409,7 +466,8 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     c->g = *g;
     c->device = device;
     c->num_sms = prop.multiProcessorCount;
-    const int max_prefill_items = ((g->max_tokens + kTileM - 1) / kTileM) * g->num_q_heads;
+    const int max_qtiles = std::max((g->max_tokens + kTileM - 1) / kTileM, 1);
+    const int max_prefill_items = max_qtiles * g->num_q_heads + kPrePartSlots;
     c->max_items = max_prefill_items + kPartSlots + std::max(g->max_decodes, 1) * g->num_kv_heads;
 
     auto bail = [&](cudaError_t e, const char *what) {
@@ -425,9 +483,13 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     const size_t part_o_bytes = (size_t)kPartSlots * kMaxRep * kHeadDim * sizeof(float);
     const size_t part_lse_bytes = (size_t)kPartSlots * kMaxRep * sizeof(float);
     const size_t merge_bytes = (size_t)std::max(g->max_decodes, 1) * g->num_kv_heads * sizeof(uint32_t);
+    const size_t pre_o_bytes = (size_t)kPrePartSlots * kTileM * kHeadDim * sizeof(float);
+    const size_t pre_lse_bytes = (size_t)kPrePartSlots * kTileM * sizeof(float);
+    const size_t pre_cnt_bytes = (((size_t)max_qtiles * g->num_q_heads * sizeof(uint32_t)) + 255) & ~size_t(255);
     c->plan_bytes = plan_capacity_bytes(c);
     const size_t plan_stride = (c->plan_bytes + 255) & ~size_t(255);
     const size_t total = part_o_bytes + part_lse_bytes + ((merge_bytes + 255) & ~size_t(255)) +
+                         pre_o_bytes + pre_lse_bytes + pre_cnt_bytes +
                          256 /*counters + err*/ + kPlanSlots * plan_stride;
     if ((e = cudaMalloc(&c->ws, total)) != cudaSuccess)
         return bail(e, "cudaMalloc(workspace)");
@@ -438,6 +500,12 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     p += part_lse_bytes;
     c->merge_cnt = reinterpret_cast<uint32_t *>(p);
     p += (merge_bytes + 255) & ~size_t(255);
+    c->pre_o = reinterpret_cast<float *>(p);
+    p += pre_o_bytes;
+    c->pre_lse = reinterpret_cast<float *>(p);
+    p += pre_lse_bytes;
+    c->pre_cnt = reinterpret_cast<uint32_t *>(p);
+    p += pre_cnt_bytes;
     c->work_cnt = reinterpret_cast<uint32_t *>(p);
     c->err = c->work_cnt + 4;
     p += 256;
@@ -450,6 +518,7 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
             return bail(e, "cudaEventCreate");
     }
     if ((e = cudaMemset(c->merge_cnt, 0, merge_bytes)) != cudaSuccess ||
+        (e = cudaMemset(c->pre_cnt, 0, pre_cnt_bytes)) != cudaSuccess ||
         (e = cudaMemset(c->work_cnt, 0, 256)) != cudaSuccess)
         return bail(e, "cudaMemset(workspace)");
     if ((e = cudaEventCreate(&c->ev_start)) != cudaSuccess ||
@@ -614,6 +683,11 @@ int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
         if (value < 0 || value > kMaxSplitKeys || value % 128)
             return fail(c, MX_EINVAL, "split keys must be 0 or a multiple of 128 up to %d", kMaxSplitKeys);
         c->split_keys_opt = (int)value;
+        return MX_OK;
+    case MX_OPT_PREFILL_PIECE_TILES:
+        if (value < 0 || value > 65535)
+            return fail(c, MX_EINVAL, "prefill piece tiles must be in [0, 65535]");
+        c->piece_tiles_opt = (int)value;
         return MX_OK;
     case MX_OPT_GRID:
         if (value < 0 || value > 65535)

@@ -21,11 +21,14 @@ constexpr int kTileN = 128;
 // Shared-memory plan (bytes, offsets from a 1024-aligned base).
 constexpr int kHalfTile = kTileM * 64 * 2;             // 128 rows x 64 bf16 = 16 KiB
 constexpr int kTileBytes = 2 * kHalfTile;              // 32 KiB
+// K tiles are released as soon as S = Q K^T has completed and V tiles after
+// P V, so K gets the deeper ring: a K load is issued ~4 tiles before use.
+constexpr int kKStages = 4;
+constexpr int kVStages = 2;
 constexpr int kSmemQ = 0;
-constexpr int kSmemK = kSmemQ + kTileBytes;            // 2 stages
-constexpr int kSmemV = kSmemK + 2 * kTileBytes;        // 2 stages
-constexpr int kSmemP = kSmemV + 2 * kTileBytes;        // 2 buffers
-constexpr int kSmemData = kSmemP + 2 * kTileBytes;     // 224 KiB
+constexpr int kSmemK = kSmemQ + kTileBytes;
+constexpr int kSmemV = kSmemK + kKStages * kTileBytes;
+constexpr int kSmemData = kSmemV + kVStages * kTileBytes;   // 224 KiB
 constexpr int kSmemMisc = kSmemData;                   // barriers etc.
 constexpr int kSmemMiscBytes = 1024;
 constexpr int kSmemTotal = kSmemData + kSmemMiscBytes + 1024;  // + alignment slack
@@ -36,9 +39,37 @@ constexpr int kDecStageBytes = 2 * kPageBytes;         // 8 KiB
 constexpr int kDecStages = 3;
 static_assert(kWarps * kDecStages * kDecStageBytes <= kSmemData, "decode ring too large");
 
+// TMEM columns: S buffers [0,128) and [128,256) (fp32), O [256,384) (fp32),
+// P buffers [384,448) and [448,512) (bf16 pairs, the A operand of P.V).
 constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kTmemO = 256;
+constexpr uint32_t kTmemP = 384;
 
 enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
+
+// Work-item encodings (int4):
+//   prefill: {ITEM_PREFILL, t | hq << 16, s | n_s << 16, partial slot base}
+//            piece s of n_s of query tile t (rows [128t, 128t+128)) of head hq;
+//            the tile's key tiles are split evenly between its n_s pieces.
+//   decode:  {ITEM_DECODE, decode index, kv head, split index}
+__host__ __device__ inline int4 prefill_item_code(int t, int hq, int s, int n_s, int part_base)
+{
+    int4 r;
+    r.x = ITEM_PREFILL;
+    r.y = t | (hq << 16);
+    r.z = s | (n_s << 16);
+    r.w = part_base;
+    return r;
+}
+__host__ __device__ inline int4 decode_item_code(int i, int h, int s)
+{
+    int4 r;
+    r.x = ITEM_DECODE;
+    r.y = i;
+    r.z = h;
+    r.w = s;
+    return r;
+}
 
 // Error bits (mirror MX_ERRBIT_* of the public header).
 constexpr uint32_t ERR_PAGE = 1u, ERR_SLOT = 2u, ERR_TIMEOUT = 4u;
@@ -69,6 +100,9 @@ struct LayerParams {
     float *part_o;         // [slot][kMaxRep][128] normalised partial outputs
     float *part_lse;       // [slot][kMaxRep] log2-sum-exp of each partial
     uint32_t *merge_cnt;   // [max_decodes * Hkv] arrival counters (self-resetting)
+    float *pre_o;          // [slot][128 rows][128] normalised prefill-piece outputs
+    float *pre_lse;        // [slot][128 rows] log2-sum-exp of each piece
+    uint32_t *pre_cnt;     // [q tiles * Hq] piece arrival counters (self-resetting)
     uint32_t *work_cnt;    // [0] next item, [1] CTAs finished (self-resetting)
     uint32_t *err;         // error word
 

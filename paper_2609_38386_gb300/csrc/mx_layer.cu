@@ -8,11 +8,13 @@
 // sees keys [0, chunk_start + j].
 //
 // Work items (built on the host, fetched with one atomic counter):
-//   ITEM_PREFILL {t, hq}:   128 chunk rows [128t, 128t+128) of query head hq
-//                           against every visible key, on tcgen05 tensor cores
-//                           (S and O accumulators in TMEM), with the append
-//                           of the tile's K/V done by the head group's first
-//                           query head.
+//   ITEM_PREFILL {t, hq, piece}: 128 chunk rows [128t, 128t+128) of query
+//                           head hq against one contiguous range of its key
+//                           tiles, on tcgen05 tensor cores (S and O
+//                           accumulators in TMEM).  A tile with several pieces
+//                           writes (O, lse) partials; the last-arriving piece
+//                           merges them.  Piece 0 of the head group's first
+//                           query head appends the tile's K/V.
 //   ITEM_DECODE  {i, h, s}: split s of decode i's keys for KV head h, all n_rep
 //                           query heads of the group at once: a split-KV
 //                           flash-decode whose partial (O, lse) is merged by
@@ -29,9 +31,10 @@ namespace mx {
 
 struct Misc {
     uint64_t bar_q;
-    uint64_t bar_kfull[2];
-    uint64_t bar_vfull[2];
-    uint64_t bar_kvempty[2];
+    uint64_t bar_kfull[kKStages];
+    uint64_t bar_kempty[kKStages];
+    uint64_t bar_vfull[kVStages];
+    uint64_t bar_vempty[kVStages];
     uint64_t bar_sfull[2];
     uint64_t bar_pfull[2];
     uint64_t bar_odone[2];
@@ -344,41 +347,52 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
 // the chunk's own keys read from the k/v inputs.
 // ---------------------------------------------------------------------------
 __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem,
-                             int t, int hq, uint32_t tile0, uint32_t item_no)
+                             int t, int hq, int kt0, int kt1, int part_slot, uint32_t tile0,
+                             uint32_t item_no)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int kvh = hq / P.n_rep;
     const int cs = P.chunk_start, p = P.p_t, nd = P.n_decodes;
     const int nA = (cs + kTileN - 1) / kTileN;
-    const int nT = nA + t + 1;
+    const int nT = kt1 - kt0;  // key tiles of this piece: global tiles kt0 + i
     const uint32_t sbase = smem_u32(smem);
-    const uint32_t sQ = sbase + kSmemQ, sK = sbase + kSmemK, sV = sbase + kSmemV,
-                   sP = sbase + kSmemP;
+    const uint32_t sQ = sbase + kSmemQ, sK = sbase + kSmemK, sV = sbase + kSmemV;
     const uint32_t bar_q = smem_u32(&misc->bar_q);
     volatile int *abort = &misc->abort;
     const uint64_t tmo = P.timeout_ns;
 
-    if (warp == 0) {
-        // ------------------------------------------------ TMA producer
-        if (lane == 0) {
+    if (warp == 0 || warp == 3) {
+        // ------------------------------------------------ TMA producers
+        // warp 0 loads Q and the K tiles, warp 3 the V tiles; each waits only
+        // on its own ring's "empty" barriers.
+        const bool isK = warp == 0;
+        if (isK && lane == 0) {
             fence_proxy_async_smem();
             mbar_expect_tx(bar_q, kTileBytes);
             tma_load_3d(sQ, &P.tm_q, bar_q, 0, hq, nd + kTileM * t);
             tma_load_3d(sQ + kHalfTile, &P.tm_q, bar_q, 64, hq, nd + kTileM * t);
         }
+        const int nst = isK ? kKStages : kVStages;
+        const uint32_t ring = isK ? sK : sV;
+        const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
+        const void *tm_in = isK ? (const void *)&P.tm_k : (const void *)&P.tm_v;
+        uint64_t *full = isK ? misc->bar_kfull : misc->bar_vfull;
+        uint64_t *empty = isK ? misc->bar_kempty : misc->bar_vempty;
         const int oob_row = P.num_pages * P.hkv * kPage;
         for (int i = 0; i < nT; ++i) {
             const uint32_t c = tile0 + i;
-            const int st = c & 1;
-            const uint32_t ph = (c >> 1) & 1;
-            const bool paged = i < nA;
+            const int st = c % nst;
+            const uint32_t ph = (c / nst) & 1;
+            const int gi = kt0 + i;
+            const bool paged = gi < nA;
             int pid_l = -1;
             if (paged && lane < 8) {
-                const int lp = i * 8 + lane;
+                const int lp = gi * 8 + lane;
                 if (lp * kPage < cs) {
                     int pid = __ldg(P.page_table + (size_t)P.prefill_seq * P.max_pages + lp);
                     if (pid < 0 || pid >= P.num_pages) {
-                        flag_error(P, ERR_PAGE);
+                        if (isK)
+                            flag_error(P, ERR_PAGE);
                         pid = -1;
                     }
                     pid_l = pid;
@@ -390,7 +404,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 pids[pg] = __shfl_sync(0xffffffffu, pid_l, pg);
             int ok = 1;
             if (lane == 0) {
-                if (!mbar_wait(smem_u32(&misc->bar_kvempty[st]), ph ^ 1, abort, tmo)) {
+                if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1, abort, tmo)) {
                     set_abort(P, misc);
                     ok = 0;
                 }
@@ -399,34 +413,22 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             if (!ok)
                 break;
             if (lane == 0) {
-                const uint32_t kf = smem_u32(&misc->bar_kfull[st]);
-                const uint32_t vf = smem_u32(&misc->bar_vfull[st]);
-                const uint32_t dk = sK + st * kTileBytes, dv = sV + st * kTileBytes;
-                mbar_expect_tx(kf, kTileBytes);
-                mbar_expect_tx(vf, kTileBytes);
+                const uint32_t fb = smem_u32(&full[st]);
+                const uint32_t dst = ring + st * kTileBytes;
+                mbar_expect_tx(fb, kTileBytes);
                 if (paged) {
 #pragma unroll
                     for (int pg = 0; pg < 8; ++pg) {
                         const int y = pids[pg] >= 0 ? (pids[pg] * P.hkv + kvh) * kPage : oob_row;
 #pragma unroll
                         for (int hf = 0; hf < 2; ++hf)
-                            tma_load_2d(dk + hf * kHalfTile + pg * 2048, &P.tm_kpool, kf, hf * 64, y);
-                    }
-#pragma unroll
-                    for (int pg = 0; pg < 8; ++pg) {
-                        const int y = pids[pg] >= 0 ? (pids[pg] * P.hkv + kvh) * kPage : oob_row;
-#pragma unroll
-                        for (int hf = 0; hf < 2; ++hf)
-                            tma_load_2d(dv + hf * kHalfTile + pg * 2048, &P.tm_vpool, vf, hf * 64, y);
+                            tma_load_2d(dst + hf * kHalfTile + pg * 2048, tm_pool, fb, hf * 64, y);
                     }
                 } else {
-                    const int z = nd + kTileN * (i - nA);
+                    const int z = nd + kTileN * (gi - nA);
 #pragma unroll
                     for (int hf = 0; hf < 2; ++hf)
-                        tma_load_3d(dk + hf * kHalfTile, &P.tm_k, kf, hf * 64, kvh, z);
-#pragma unroll
-                    for (int hf = 0; hf < 2; ++hf)
-                        tma_load_3d(dv + hf * kHalfTile, &P.tm_v, vf, hf * 64, kvh, z);
+                        tma_load_3d(dst + hf * kHalfTile, tm_in, fb, hf * 64, kvh, z);
                 }
             }
         }
@@ -437,17 +439,17 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             tc_fence_after();
             auto issue_pv = [&](int i) -> bool {
                 const uint32_t c = tile0 + i;
-                const int st = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
+                const int st = c % kVStages;
+                const uint32_t ph = (c / kVStages) & 1;
                 if (!mbar_wait(smem_u32(&misc->bar_pfull[c & 1]), (c >> 1) & 1, abort, tmo))
                     return false;
                 if (!mbar_wait(smem_u32(&misc->bar_vfull[st]), ph, abort, tmo))
                     return false;
                 const uint32_t dv = sV + st * kTileBytes;
-                if (i == nA - 1 && (cs % kTileN) != 0) {
+                if (kt0 + i == nA - 1 && (cs % kTileN) != 0) {
                     // keys [cs, end of that page) of the last paged tile are not
                     // cached yet: clear their value rows (later pages are zero).
-                    const int r0 = cs - i * kTileN;
+                    const int r0 = cs - (kt0 + i) * kTileN;
                     const int r1 = min(kTileN, (r0 + kPage - 1) / kPage * kPage);
                     for (int r = r0; r < r1; ++r)
                         for (int hf = 0; hf < 2; ++hf)
@@ -459,21 +461,20 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                     fence_proxy_async_smem();
                 }
                 tc_fence_after();
-                const uint32_t pb = sP + (c & 1) * kTileBytes;
+                const uint32_t pa = tmem + kTmemP + (c & 1) * 64;  // P_c: 8 columns per 16 keys
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
-                    const uint64_t a = smem_desc(pb + (kk >> 2) * kHalfTile + (kk & 3) * 32, 16, 1024, kSwz128);
                     const uint64_t b = smem_desc(dv + kk * 2048, kHalfTile, 1024, kSwz128);
-                    tc_mma_ss(tmem + 256, a, b, kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
+                    tc_mma_ts(tmem + kTmemO, pa + kk * 8, b, kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
                 }
                 tc_commit(smem_u32(&misc->bar_odone[c & 1]));
-                tc_commit(smem_u32(&misc->bar_kvempty[st]));
+                tc_commit(smem_u32(&misc->bar_vempty[st]));
                 return true;
             };
             for (int i = 0; ok && i < nT; ++i) {
                 const uint32_t c = tile0 + i;
-                const int st = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
+                const int st = c % kKStages;
+                const uint32_t ph = (c / kKStages) & 1;
                 if (!mbar_wait(smem_u32(&misc->bar_kfull[st]), ph, abort, tmo)) {
                     ok = false;
                     break;
@@ -487,6 +488,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                     tc_mma_ss(tmem + (c & 1) * 128, a, b, kIdescS, kk > 0 ? 1u : 0u);
                 }
                 tc_commit(smem_u32(&misc->bar_sfull[c & 1]));
+                tc_commit(smem_u32(&misc->bar_kempty[st]));
                 if (i > 0 && !issue_pv(i - 1))
                     ok = false;
             }
@@ -496,28 +498,47 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 set_abort(P, misc);
         }
         __syncwarp();
-    } else if (warp < 4) {
+    } else if (warp == 2) {
         // ------------------------------------------------ chunk KV append
-        if (hq % P.n_rep == 0) {
-            const int j0 = kTileM * t;
-            const int ntok = min(kTileM, p - j0);
-            for (int e = (warp - 2) * 32 + lane; e < ntok * 32; e += 64) {
-                const int tok = nd + j0 + e / 32, w = e % 32;
-                const int slot = __ldg(P.slots + tok);
-                if (slot < 0)
-                    continue;
-                if (slot >= P.num_pages * kPage) {
-                    flag_error(P, ERR_SLOT);
-                    continue;
+        // The n_rep query heads of a KV head share its 128 tokens: head r of
+        // the group appends tokens [r*128/n_rep, (r+1)*128/n_rep) of the tile.
+        // 16 tokens per round so that 16 loads per lane are in flight.
+        if (kt0 == 0) {
+            const int per = kTileM / P.n_rep;
+            const int j0 = kTileM * t + (hq % P.n_rep) * per;
+            const int ntok = min(per, p - j0);
+            constexpr int U = 16;
+            const int c16 = lane & 15;
+            const bool isv = lane >= 16;
+            const uint16_t *src_base = isv ? P.v : P.k;
+            uint16_t *dst_base = isv ? P.v_pool : P.k_pool;
+            for (int tb = 0; tb < ntok; tb += U) {
+                int my_slot = -1;
+                if (lane < U && tb + lane < ntok)
+                    my_slot = __ldg(P.slots + nd + j0 + tb + lane);
+                uint4 val[U];
+                int sl[U];
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    sl[u] = __shfl_sync(0xffffffffu, my_slot, u);
+                    if (tb + u < ntok && sl[u] >= 0 && sl[u] < P.num_pages * kPage) {
+                        const size_t src = ((size_t)(nd + j0 + tb + u) * P.hkv + kvh) * kHeadDim;
+                        val[u] = __ldg(reinterpret_cast<const uint4 *>(src_base + src) + c16);
+                    }
                 }
-                const size_t dst = (((size_t)(slot / kPage) * P.hkv + kvh) * kPage + slot % kPage) * kHeadDim;
-                const size_t src = ((size_t)tok * P.hkv + kvh) * kHeadDim;
-                if (w < 16)
-                    reinterpret_cast<uint4 *>(P.k_pool + dst)[w] =
-                        __ldg(reinterpret_cast<const uint4 *>(P.k + src) + w);
-                else
-                    reinterpret_cast<uint4 *>(P.v_pool + dst)[w - 16] =
-                        __ldg(reinterpret_cast<const uint4 *>(P.v + src) + (w - 16));
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    if (tb + u >= ntok || sl[u] < 0)
+                        continue;
+                    if (sl[u] >= P.num_pages * kPage) {
+                        if (lane == 0)
+                            flag_error(P, ERR_SLOT);
+                        continue;
+                    }
+                    const size_t dst =
+                        (((size_t)(sl[u] / kPage) * P.hkv + kvh) * kPage + sl[u] % kPage) * kHeadDim;
+                    reinterpret_cast<uint4 *>(dst_base + dst)[c16] = val[u];
+                }
             }
         }
     } else {
@@ -542,27 +563,42 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             for (int gq = 0; gq < 4; ++gq)
                 tmem_ld32(tl + sb * 128 + 32 * gq, *reinterpret_cast<uint32_t(*)[32]>(&sv[32 * gq]));
             tmem_wait_ld();
-            const int nvalid = i < nA ? min(kTileN, cs - i * kTileN)
-                                      : min(kTileN, j - kTileN * (i - nA) + 1);
-            float mx = neg_inf();
+            const int gi = kt0 + i;
+            const int nvalid = gi < nA ? min(kTileN, cs - gi * kTileN)
+                                       : min(kTileN, j - kTileN * (gi - nA) + 1);
+            if (nvalid < kTileN) {  // boundary tiles only: masked keys -> -inf
 #pragma unroll
-            for (int cc = 0; cc < 128; ++cc) {
-                const float x = cc < nvalid ? __uint_as_float(sv[cc]) * sl : neg_inf();
-                sv[cc] = __float_as_uint(x);
-                mx = fmaxf(mx, x);
+                for (int cc = 0; cc < 128; ++cc)
+                    if (cc >= nvalid)
+                        sv[cc] = 0xFF800000u;
             }
-            const float m_new = fmaxf(m_run, mx);
+            // row max of the raw scores (the scale is positive), 8 chains
+            float mx8[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                mx8[u] = __uint_as_float(sv[u]);
+#pragma unroll
+            for (int cc = 8; cc < 128; ++cc)
+                mx8[cc & 7] = fmaxf(mx8[cc & 7], __uint_as_float(sv[cc]));
+            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+            const float m_new = fmaxf(m_run, mx * sl);   // log2 domain
             const bool rescale = m_new > m_run + 8.0f;
             const float m_use = rescale ? m_new : m_run;
-            float rs = 0.f;
+            const float nm = -m_use;
+            float rs8[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                rs8[u] = 0.f;
             uint32_t pk[64];
 #pragma unroll
             for (int cc = 0; cc < 64; ++cc) {
-                const float e0 = ex2(__uint_as_float(sv[2 * cc]) - m_use);
-                const float e1 = ex2(__uint_as_float(sv[2 * cc + 1]) - m_use);
-                rs += e0 + e1;
+                const float e0 = ex2(fmaf(__uint_as_float(sv[2 * cc]), sl, nm));
+                const float e1 = ex2(fmaf(__uint_as_float(sv[2 * cc + 1]), sl, nm));
+                rs8[cc & 7] += e0 + e1;
                 pk[cc] = pack_bf16(e0, e1);
             }
+            const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
             // P buffer (c & 1) was last read by tile c - 2's PV.
             if (i >= 2 && !mbar_wait(smem_u32(&misc->bar_odone[c & 1]), ((c - 2) >> 1) & 1, abort, tmo)) {
                 ok = false;
@@ -579,31 +615,22 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
 #pragma unroll
                 for (int gq = 0; gq < 4; ++gq) {
                     uint32_t o[32];
-                    tmem_ld32(tl + 256 + 32 * gq, o);
+                    tmem_ld32(tl + kTmemO + 32 * gq, o);
                     tmem_wait_ld();
 #pragma unroll
                     for (int x = 0; x < 32; ++x)
                         o[x] = __float_as_uint(__uint_as_float(o[x]) * alpha);
-                    tmem_st32(tl + 256 + 32 * gq, o);
+                    tmem_st32(tl + kTmemO + 32 * gq, o);
                 }
                 tmem_wait_st();
                 l_run *= alpha;
             }
             l_run += rs;
             m_run = m_use;
-            // P row r into the 128-byte-swizzled K-major tile
-            const uint32_t prow = sP + (c & 1) * kTileBytes + r * 128;
-#pragma unroll
-            for (int hf = 0; hf < 2; ++hf)
-#pragma unroll
-                for (int cc = 0; cc < 8; ++cc) {
-                    const int w0 = hf * 32 + cc * 4;
-                    asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(
-                                     prow + hf * kHalfTile + ((cc ^ (r & 7)) << 4)),
-                                 "r"(pk[w0]), "r"(pk[w0 + 1]), "r"(pk[w0 + 2]), "r"(pk[w0 + 3])
-                                 : "memory");
-                }
-            fence_proxy_async_smem();
+            // P row r (bf16 pairs) into TMEM lane r, the A operand of P.V
+            tmem_st32(tl + kTmemP + (c & 1) * 64, *reinterpret_cast<const uint32_t(*)[32]>(&pk[0]));
+            tmem_st32(tl + kTmemP + (c & 1) * 64 + 32, *reinterpret_cast<const uint32_t(*)[32]>(&pk[32]));
+            tmem_wait_st();
             tc_fence_before();
             mbar_arrive(smem_u32(&misc->bar_pfull[c & 1]));
         }
@@ -614,6 +641,26 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         }
         if (!ok) {
             set_abort(P, misc);
+        } else if (part_slot >= 0) {
+            // one piece of a split tile: normalised partial O and its lse
+            tc_fence_after();
+            const float inv = 1.0f / l_run;
+            float *prow = P.pre_o + ((size_t)part_slot * kTileM + r) * kHeadDim;
+#pragma unroll
+            for (int gq = 0; gq < 4; ++gq) {
+                uint32_t o[32];
+                tmem_ld32(tl + kTmemO + 32 * gq, o);
+                tmem_wait_ld();
+#pragma unroll
+                for (int x = 0; x < 8; ++x)
+                    reinterpret_cast<float4 *>(prow + 32 * gq)[x] =
+                        make_float4(__uint_as_float(o[4 * x]) * inv, __uint_as_float(o[4 * x + 1]) * inv,
+                                    __uint_as_float(o[4 * x + 2]) * inv, __uint_as_float(o[4 * x + 3]) * inv);
+            }
+            float lg;
+            asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(lg) : "f"(l_run));
+            P.pre_lse[(size_t)part_slot * kTileM + r] = m_run + lg;
+            __threadfence();
         } else {
             tc_fence_after();
             const float inv = 1.0f / l_run;
@@ -621,7 +668,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
 #pragma unroll
             for (int gq = 0; gq < 4; ++gq) {
                 uint32_t o[32];
-                tmem_ld32(tl + 256 + 32 * gq, o);
+                tmem_ld32(tl + kTmemO + 32 * gq, o);
                 tmem_wait_ld();
                 if (j < p) {
 #pragma unroll
@@ -639,6 +686,64 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
     }
 }
 
+// Merge the n_s pieces of prefill tile (t, hq) if this CTA's piece arrived
+// last (no waiting): out = sum_s w_s O_s / sum_s w_s, w_s = 2^(lse_s - max).
+__device__ void prefill_merge(const LayerParams &P, Misc *misc, int t, int hq, int n_s,
+                              int part_base)
+{
+    const int tid = threadIdx.x;
+    if (tid == 0) {
+        const uint32_t prev = atomicAdd(P.pre_cnt + t * P.hq + hq, 1u);
+        misc->last = (prev == (uint32_t)(n_s - 1)) ? 1 : 0;
+    }
+    __syncthreads();
+    if (misc->last) {
+        __threadfence();
+        const int r = tid >> 1, half = tid & 1;
+        const int j = kTileM * t + r;
+        if (j < P.p_t) {
+            float M = neg_inf();
+            for (int s = 0; s < n_s; ++s)
+                M = fmaxf(M, __ldcg(P.pre_lse + (size_t)(part_base + s) * kTileM + r));
+            float W = 0.f;
+            for (int s = 0; s < n_s; ++s)
+                W += ex2(__ldcg(P.pre_lse + (size_t)(part_base + s) * kTileM + r) - M);
+            const float inv = 1.0f / W;
+            for (int sub = 0; sub < 2; ++sub) {
+                const int d0 = half * 64 + sub * 32;
+                float acc[32];
+#pragma unroll
+                for (int x = 0; x < 32; ++x)
+                    acc[x] = 0.f;
+                for (int s = 0; s < n_s; ++s) {
+                    const float w = ex2(__ldcg(P.pre_lse + (size_t)(part_base + s) * kTileM + r) - M);
+                    const float4 *src = reinterpret_cast<const float4 *>(
+                        P.pre_o + ((size_t)(part_base + s) * kTileM + r) * kHeadDim + d0);
+#pragma unroll
+                    for (int x = 0; x < 8; ++x) {
+                        const float4 v = __ldcg(src + x);
+                        acc[4 * x] += w * v.x;
+                        acc[4 * x + 1] += w * v.y;
+                        acc[4 * x + 2] += w * v.z;
+                        acc[4 * x + 3] += w * v.w;
+                    }
+                }
+                uint4 *dst = reinterpret_cast<uint4 *>(
+                    P.out + ((size_t)(P.n_decodes + j) * P.hq + hq) * kHeadDim + d0);
+#pragma unroll
+                for (int x = 0; x < 4; ++x)
+                    dst[x] = make_uint4(pack_bf16(acc[8 * x] * inv, acc[8 * x + 1] * inv),
+                                        pack_bf16(acc[8 * x + 2] * inv, acc[8 * x + 3] * inv),
+                                        pack_bf16(acc[8 * x + 4] * inv, acc[8 * x + 5] * inv),
+                                        pack_bf16(acc[8 * x + 6] * inv, acc[8 * x + 7] * inv));
+            }
+        }
+        if (tid == 0)
+            P.pre_cnt[t * P.hq + hq] = 0u;
+    }
+    __syncthreads();
+}
+
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_constant__ LayerParams P)
 {
@@ -650,10 +755,15 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
 
     if (tid == 0) {
         mbar_init(smem_u32(&misc->bar_q), 1);
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < kKStages; ++b) {
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
+            mbar_init(smem_u32(&misc->bar_kempty[b]), 1);
+        }
+        for (int b = 0; b < kVStages; ++b) {
             mbar_init(smem_u32(&misc->bar_vfull[b]), 1);
-            mbar_init(smem_u32(&misc->bar_kvempty[b]), 1);
+            mbar_init(smem_u32(&misc->bar_vempty[b]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&misc->bar_sfull[b]), 1);
             mbar_init(smem_u32(&misc->bar_pfull[b]), 128);
             mbar_init(smem_u32(&misc->bar_odone[b]), 1);
@@ -687,12 +797,21 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         if (tid == 0)
             misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
         const int4 it = P.items[idx];
+        int merge_t = -1, merge_hq = 0, merge_ns = 1;
         if (it.x == ITEM_PREFILL) {
-            prefill_item(P, smem, misc, tmem, it.y, it.z,
-                         tile_cnt, item_no);
-            const int nA = (P.chunk_start + kTileN - 1) / kTileN;
-            tile_cnt += nA + it.y + 1;
+            const int t = it.y & 0xFFFF, hq = it.y >> 16;
+            const int s = it.z & 0xFFFF, ns = it.z >> 16;
+            const int nT = (P.chunk_start + kTileN - 1) / kTileN + t + 1;
+            const int kt0 = (int)((long long)s * nT / ns), kt1 = (int)((long long)(s + 1) * nT / ns);
+            prefill_item(P, smem, misc, tmem, t, hq, kt0, kt1, ns > 1 ? it.w + s : -1, tile_cnt,
+                         item_no);
+            tile_cnt += kt1 - kt0;
             item_no += 1;
+            if (ns > 1) {
+                merge_t = t;
+                merge_hq = hq;
+                merge_ns = ns;
+            }
         } else {
             decode_item(P, smem, misc, it.y, it.z, it.w);
         }
@@ -700,6 +819,8 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
+        if (merge_t >= 0 && !misc->abort)
+            prefill_merge(P, misc, merge_t, merge_hq, merge_ns, it.w);
         buf ^= 1;
     }
 

@@ -222,7 +222,7 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     int n = 0;
     for (int t = n_qt - 1; t >= 0; --t)
         for (int h = 0; h < hq; ++h)
-            items[n++] = make_int4(ITEM_PREFILL, t, h, 0);
+            items[n++] = prefill_item_code(t, h, 0, 1, 0);
     const int n_prefill = n;
     int part = 0;
     for (int i = 0; i < nd; ++i) {
@@ -239,14 +239,14 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
         const int ns = dec[i].n_splits;
         for (int h = 0; h < hkv; ++h)
             for (int s = 0; s < ns - 1; ++s)
-                items[n++] = make_int4(ITEM_DECODE, i, h, s);
+                items[n++] = decode_item_code(i, h, s);
     }
     const int tail0 = n;
     for (int i = 0; i < nd; ++i)
         for (int h = 0; h < hkv; ++h)
-            items[n++] = make_int4(ITEM_DECODE, i, h, dec[i].n_splits - 1);
+            items[n++] = decode_item_code(i, h, dec[i].n_splits - 1);
     std::stable_sort(items + tail0, items + n, [&](const int4 &a, const int4 &c) {
-        const int ka = dec[a.y].ctx + 1 - (dec[a.y].n_splits - 1) * split;
+        const int ka = dec[a.y].ctx + 1 - (dec[a.y].n_splits - 1) * split;   // .y: decode index
         const int kc = dec[c.y].ctx + 1 - (dec[c.y].n_splits - 1) * split;
         return ka > kc;
     });

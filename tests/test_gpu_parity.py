@@ -209,3 +209,33 @@ def test_iteration_returns_device_time():
     _ok(ref)
     np.testing.assert_array_equal(devs[1]["out"].cpu().numpy(), devs[0]["out"].cpu().numpy())
     ctx.close()
+
+
+@pytest.mark.parametrize("piece", [1, 2, 3, 5])
+@pytest.mark.parametrize("cs,p", [(0, 384), (1000, 300), (77, 200)])
+def test_prefill_key_pieces(piece, cs, p):
+    """Prefill tiles split along keys into pieces merged by log-sum-exp."""
+    from paper_2609_38386_gb300 import MX_OPT_PREFILL_PIECE_TILES
+    case = Case(32, [900, 3], chunk_start=cs, p_t=p, seed=piece * 7 + cs)
+    res = case.run_gpu(options={MX_OPT_PREFILL_PIECE_TILES: piece})
+    _ok(case.check(res))
+
+
+def test_prefill_auto_pieces_long_context():
+    # a short chunk deep into a long prompt: the planner splits its tiles
+    case = Case(16, [2000, 40], chunk_start=6000, p_t=200, seed=8)
+    res = case.run_gpu()
+    assert res["plan"]["n_prefill_items"] > 2 * 16
+    _ok(case.check(res))
+
+
+def test_prefill_pieces_deterministic_and_reusable():
+    from paper_2609_38386_gb300 import MX_OPT_PREFILL_PIECE_TILES
+    case = Case(16, [], chunk_start=700, p_t=256, seed=9)
+    ctx = case.make_context()
+    ctx.set_option(MX_OPT_PREFILL_PIECE_TILES, 2)
+    r1 = case.run_gpu(ctx=ctx)
+    r2 = case.run_gpu(ctx=ctx)        # counters reset by the previous launch
+    np.testing.assert_array_equal(r1["out"], r2["out"])
+    _ok(case.check(r2))
+    ctx.close()
