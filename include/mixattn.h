@@ -184,7 +184,7 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  * Same operation, layouts and descriptor as mx_mixed_attention (geom gives
  * the geometry a context would hold; max_tokens / max_decodes are ignored).
  * Its scratch (work list, split partials, counters, error word) is one fixed
- * 4.24 MiB device array built into the library, which every GPU that loads
+ * 4.11 MiB device array built into the library, which every GPU that loads
  * the library holds until the process exits.  Limits: n_decodes <= 256,
  * at most 4096 work items (prefill tiles = ceil(p_t / 128) * Hq, plus decode
  * splits), at most 1024 split partials, num_kv_heads <= 16; a request beyond

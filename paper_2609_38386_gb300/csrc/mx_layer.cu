@@ -558,47 +558,38 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 break;
             }
             tc_fence_after();
-            uint32_t sv[128];
-#pragma unroll
-            for (int gq = 0; gq < 4; ++gq)
-                tmem_ld32(tl + sb * 128 + 32 * gq, *reinterpret_cast<uint32_t(*)[32]>(&sv[32 * gq]));
-            tmem_wait_ld();
             const int gi = kt0 + i;
             const int nvalid = gi < nA ? min(kTileN, cs - gi * kTileN)
                                        : min(kTileN, j - kTileN * (gi - nA) + 1);
-            if (nvalid < kTileN) {  // boundary tiles only: masked keys -> -inf
-#pragma unroll
-                for (int cc = 0; cc < 128; ++cc)
-                    if (cc >= nvalid)
-                        sv[cc] = 0xFF800000u;
-            }
-            // row max of the raw scores (the scale is positive), 8 chains
+            // Pass 1: row max of the raw scores (the scale is positive) over
+            // the two 64-column halves of S, 8 independent chains.  S is read
+            // from TMEM twice (here and in pass 2) to keep only 64 scores live.
             float mx8[8];
 #pragma unroll
             for (int u = 0; u < 8; ++u)
-                mx8[u] = __uint_as_float(sv[u]);
+                mx8[u] = neg_inf();
 #pragma unroll
-            for (int cc = 8; cc < 128; ++cc)
-                mx8[cc & 7] = fmaxf(mx8[cc & 7], __uint_as_float(sv[cc]));
+            for (int half = 0; half < 2; ++half) {
+                uint32_t sv[64];
+                tmem_ld32(tl + sb * 128 + 64 * half, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+                tmem_ld32(tl + sb * 128 + 64 * half + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+                tmem_wait_ld();
+                if (nvalid < kTileN) {  // boundary tiles only: masked keys -> -inf
+#pragma unroll
+                    for (int cc = 0; cc < 64; ++cc)
+                        if (64 * half + cc >= nvalid)
+                            sv[cc] = 0xFF800000u;
+                }
+#pragma unroll
+                for (int cc = 0; cc < 64; ++cc)
+                    mx8[cc & 7] = fmaxf(mx8[cc & 7], __uint_as_float(sv[cc]));
+            }
             const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                                    fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
             const float m_new = fmaxf(m_run, mx * sl);   // log2 domain
             const bool rescale = m_new > m_run + 8.0f;
             const float m_use = rescale ? m_new : m_run;
             const float nm = -m_use;
-            float rs8[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u)
-                rs8[u] = 0.f;
-            uint32_t pk[64];
-#pragma unroll
-            for (int cc = 0; cc < 64; ++cc) {
-                const float e0 = ex2(fmaf(__uint_as_float(sv[2 * cc]), sl, nm));
-                const float e1 = ex2(fmaf(__uint_as_float(sv[2 * cc + 1]), sl, nm));
-                rs8[cc & 7] += e0 + e1;
-                pk[cc] = pack_bf16(e0, e1);
-            }
-            const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
             // P buffer (c & 1) was last read by tile c - 2's PV.
             if (i >= 2 && !mbar_wait(smem_u32(&misc->bar_odone[c & 1]), ((c - 2) >> 1) & 1, abort, tmo)) {
                 ok = false;
@@ -625,11 +616,37 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 tmem_wait_st();
                 l_run *= alpha;
             }
+            // Pass 2: p = 2^(s*scale - m) as bf16 pairs into TMEM lane r (the A
+            // operand of P.V), and the row sum with 8 chains.
+            float rs8[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                rs8[u] = 0.f;
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                uint32_t sv[64];
+                tmem_ld32(tl + sb * 128 + 64 * half, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+                tmem_ld32(tl + sb * 128 + 64 * half + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+                tmem_wait_ld();
+                if (nvalid < kTileN) {
+#pragma unroll
+                    for (int cc = 0; cc < 64; ++cc)
+                        if (64 * half + cc >= nvalid)
+                            sv[cc] = 0xFF800000u;
+                }
+                uint32_t pk[32];
+#pragma unroll
+                for (int cc = 0; cc < 32; ++cc) {
+                    const float e0 = ex2(fmaf(__uint_as_float(sv[2 * cc]), sl, nm));
+                    const float e1 = ex2(fmaf(__uint_as_float(sv[2 * cc + 1]), sl, nm));
+                    rs8[cc & 7] += e0 + e1;
+                    pk[cc] = pack_bf16(e0, e1);
+                }
+                tmem_st32(tl + kTmemP + (c & 1) * 64 + 32 * half, pk);
+            }
+            const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
             l_run += rs;
             m_run = m_use;
-            // P row r (bf16 pairs) into TMEM lane r, the A operand of P.V
-            tmem_st32(tl + kTmemP + (c & 1) * 64, *reinterpret_cast<const uint32_t(*)[32]>(&pk[0]));
-            tmem_st32(tl + kTmemP + (c & 1) * 64 + 32, *reinterpret_cast<const uint32_t(*)[32]>(&pk[32]));
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(smem_u32(&misc->bar_pfull[c & 1]));

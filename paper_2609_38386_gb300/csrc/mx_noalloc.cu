@@ -12,7 +12,7 @@
 // in one fixed file-scope device array that the module loader places in
 // device memory together with the code.
 //
-// Limits (the size of that array, 4.24 MiB): at most 256 decodes, 4096 work
+// Limits (the size of that array, 4.11 MiB): at most 256 decodes, 4096 work
 // items, 1024 decode split partials, 16 KV heads.  Larger requests are
 // rejected with MX_ECAPACITY before anything is enqueued.
 //
