@@ -235,3 +235,29 @@ def compare_rows(case, res, rows):
     if not np.all(np.isfinite(got)):
         return {"max_abs": float("inf"), "mean_abs": float("inf")}
     return {"max_abs": float(err.max()), "mean_abs": float(err.mean())}
+
+
+def check_pages(case, d, n_untouched=32, seed=0):
+    """KV pages after the call: every page the append touched equals its
+    initial contents with the new rows written at their slots; a random
+    sample of untouched pages is unchanged.  Returns the number of pages
+    compared."""
+    import torch
+    ps = case.geom.page_size
+    valid = case.slots >= 0
+    toks = np.nonzero(valid)[0]
+    sl = case.slots[valid].astype(np.int64)
+    touched = np.unique(sl // ps)
+    rng = np.random.default_rng(seed)
+    others = np.setdiff1d(np.arange(case.layout.num_pages), touched)
+    untouched = rng.choice(others, size=min(n_untouched, len(others)), replace=False)
+    pages = np.concatenate([touched, untouched])
+    kp, vp = case.pages0(pages)
+    where = np.searchsorted(touched, sl // ps)
+    kp[where, :, sl % ps, :] = case.k[toks]
+    vp[where, :, sl % ps, :] = case.v[toks]
+    sel = torch.from_numpy(pages).to(d["k_pool"].device)
+    got_k = d["k_pool"][sel].cpu().numpy().view(np.uint16)
+    got_v = d["v_pool"][sel].cpu().numpy().view(np.uint16)
+    assert np.array_equal(got_k, kp) and np.array_equal(got_v, vp), "KV pages differ"
+    return len(pages)
