@@ -316,6 +316,106 @@ def cpu_baseline(cfg, which="heavy"):
             "kind": "oracle", "sample": desc, "seconds": dt}
 
 
+# ------------------------------------------------------------- DLFP trace
+class TraceEngine:
+    """Device state for an open-loop trace: per-layer pools with pages for
+    every request's prompt and output, a page table with one row per request,
+    q/k/v/out buffers sized for one iteration's token budget, and the
+    completion-timed iteration call (`execute(plan) -> device us`)."""
+
+    def __init__(self, requests, n_layers, hq, device, seed, budget, max_seqs):
+        import torch
+
+        import synth
+        from paper_2609_38386_gb300 import Context
+        from synth import device as sdev
+        from synth import workload as wl
+        self.geom = g = wl.Geometry(hq)
+        caps = [r.prompt + r.output for r in requests]
+        self.layout = lay = wl.make_layout(g, caps, seed=seed + 7)
+        self.max_tok = budget + max_seqs
+        self.ctx = Context(num_q_heads=hq, num_kv_heads=g.hkv, num_pages=lay.num_pages,
+                           num_seqs=lay.num_seqs, max_pages_per_seq=lay.max_pages,
+                           max_tokens=self.max_tok, max_decodes=max_seqs,
+                           device=device.index or 0)
+        self.page_table = torch.from_numpy(lay.page_table).to(device)
+        self.slots_h = torch.empty(self.max_tok, dtype=torch.int32, pin_memory=True)
+        self.slots_d = torch.empty(self.max_tok, dtype=torch.int32, device=device)
+        self.keep = []
+        bufs = []
+        for l in range(n_layers):
+            kp = torch.empty(lay.pool_shape(), dtype=torch.int16, device=device)
+            vp = torch.empty_like(kp)
+            sdev.fill_(kp, wl.pool_base(seed, l, synth.STREAM_KPOOL))
+            sdev.fill_(vp, wl.pool_base(seed, l, synth.STREAM_VPOOL))
+            q = torch.empty((self.max_tok, hq, g.head_dim), dtype=torch.int16, device=device)
+            k = torch.empty((self.max_tok, g.hkv, g.head_dim), dtype=torch.int16, device=device)
+            v = torch.empty_like(k)
+            for t, kind in ((q, synth.STREAM_Q), (k, synth.STREAM_K), (v, synth.STREAM_V)):
+                sdev.fill_(t, synth.stream_base(seed, synth.stream_id(l, kind, 7)))
+            out = torch.empty_like(q)
+            self.keep.append((kp, vp, q, k, v, out))
+            bufs.append(self.ctx.make_bufs(q, k, v, kp, vp, out))
+        self.layers = self.ctx.layer_array(bufs)
+        torch.cuda.synchronize(device)
+        self.iterations = 0
+
+    def execute(self, plan):
+        import numpy as np
+        lay = self.layout
+        parts = [lay.slot(rid, ctx)[None] for rid, ctx in zip(plan.decode_ids, plan.decode_ctx)]
+        if plan.p_t:
+            parts.append(lay.slot(plan.prefill_id,
+                                  np.arange(plan.chunk_start, plan.chunk_start + plan.p_t)))
+        n = len(plan.decode_ids) + plan.p_t
+        if n:
+            self.slots_h[:n].copy_(__import__("torch").from_numpy(np.concatenate(parts)))
+            self.slots_d[:n].copy_(self.slots_h[:n], non_blocking=True)
+        desc = self.ctx.make_desc(decode_seq_ids=plan.decode_ids, decode_ctx_lens=plan.decode_ctx,
+                                  prefill_seq_id=plan.prefill_id, chunk_start=plan.chunk_start,
+                                  p_t=plan.p_t, page_table=self.page_table, slots=self.slots_d)
+        self.iterations += 1
+        return self.ctx.iteration(desc, self.layers)
+
+
+def trace_measure(device, seeds=(801, 802, 803), n_layers=28, hq=16, budget=8192,
+                  max_seqs=64, fixed_cap=2048):
+    """Config 5: the completion-timed DLFP loop against a fixed chunk cap on
+    seeded open-loop traces (§3.1 Eq. 2 with L_t = device-completion time)."""
+    import numpy as np
+    import torch
+
+    from paper_2609_38386_gb300 import dlfp
+    # t_ref: 16 decodes at context 1024 beside a 2048-token chunk at position 0
+    cal_reqs = [dlfp.Request(i, 0.0, 1025, 2) for i in range(16)] + [dlfp.Request(16, 0.0, 2048, 1)]
+    eng = TraceEngine(cal_reqs, n_layers, hq, device, 0, budget, max_seqs)
+    cal = dlfp.IterationPlan(list(range(16)), [1024] * 16, 16, 0, 2048, None)
+    for _ in range(3):
+        eng.execute(cal)
+    t_ref = float(np.median([eng.execute(cal) for _ in range(7)]))
+    del eng
+    torch.cuda.empty_cache()
+    result = {"t_ref_us": t_ref, "mean_interarrival_us": 20 * t_ref, "target_us": t_ref,
+              "fixed_cap": fixed_cap, "seeds": {}}
+    red = []
+    for seed in seeds:
+        spec = dlfp.TraceSpec(mean_interarrival=20 * t_ref, seed=seed)
+        eng = TraceEngine(spec.requests(), n_layers, hq, device, seed, budget, max_seqs)
+        per = {}
+        for name in ("fixed", "dlfp"):
+            ctl = dlfp.FixedCap(fixed_cap) if name == "fixed" else dlfp.DLFPController(t_ref)
+            sch = dlfp.Scheduler(spec.requests(), ctl, max_seqs=max_seqs, budget=budget)
+            t0 = time.perf_counter()
+            per[name] = sch.run(eng.execute)
+            per[name]["wall_s"] = time.perf_counter() - t0
+        red.append(1 - per["dlfp"]["itl_p99"] / per["fixed"]["itl_p99"])
+        result["seeds"][str(seed)] = per
+        del eng
+        torch.cuda.empty_cache()
+    result["mean_itl_p99_reduction"] = float(np.mean(red))
+    return result
+
+
 # ------------------------------------------------------------------- main
 def main():
     ap = argparse.ArgumentParser()
@@ -329,6 +429,8 @@ def main():
     ap.add_argument("--profile-chunk", type=int, default=2048)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--workload", default="sweep", choices=["sweep", "trace"],
+                    help="trace: the completion-timed DLFP loop vs a fixed chunk cap")
     args = ap.parse_args()
 
     ws, rank, local = dist_setup()
@@ -367,6 +469,15 @@ def main():
         return
 
     import torch
+    if args.workload == "trace":
+        if rank == 0:
+            device = torch.device("cuda", local)
+            torch.cuda.set_device(device)
+            res = trace_measure(device)
+            print(json.dumps({"metric": "open-loop trace: per-iteration device us P50/P99 and "
+                              "ITL/TTFT, completion-timed DLFP vs fixed chunk cap",
+                              "workload": "qwen3-0.6b-attn-28L-poisson-trace", **res}))
+        return
     if ws > 1:
         import torch.distributed as dist
         torch.cuda.set_device(local)
