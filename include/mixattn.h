@@ -168,6 +168,10 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
 #define MX_OPT_SPLIT_KEYS 1
 #define MX_OPT_GRID 2
 #define MX_OPT_PREFILL_PIECE_TILES 3
+/* MX_OPT_PDL: 1 (default) launches each layer kernel with programmatic
+ * dependent launch, so the next layer's CTAs start their set-up on SMs the
+ * previous layer has freed; 0 = ordinary stream order. */
+#define MX_OPT_PDL 4
 int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 
 /* Number of work items and decode split length chosen for the last planned

@@ -21,6 +21,7 @@ ERRORS = {-1: "MX_EINVAL", -2: "MX_ERANGE_PAGE", -3: "MX_ERANGE_SLOT", -4: "MX_E
 MX_OPT_SPLIT_KEYS = 1
 MX_OPT_GRID = 2
 MX_OPT_PREFILL_PIECE_TILES = 3
+MX_OPT_PDL = 4
 
 # Names every C-ABI build must export (the declarations of include/mixattn.h).
 EXPORTS = ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",

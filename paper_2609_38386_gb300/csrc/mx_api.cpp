@@ -16,7 +16,7 @@
 
 namespace mx {
 cudaError_t init_layer_kernel();
-cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream);
+cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream, bool pdl);
 cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int num_pages,
                              const uint16_t *k, const uint16_t *v, uint16_t *k_pool,
                              uint16_t *v_pool, uint32_t *err, cudaStream_t stream);
@@ -68,6 +68,7 @@ struct mx_ctx {
     int split_keys_opt = 0;
     int grid_opt = 0;
     int piece_tiles_opt = 0;
+    bool pdl = true;  // programmatic dependent launch between layer kernels
     // last plan
     int last_items = 0, last_split = 0, last_prefill_items = 0, last_piece_tiles = 0;
     std::string last_error;
@@ -602,7 +603,7 @@ int mx_mixed_attention(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b,
     LayerParams P;
     if ((rc = make_params(c, d, b, pl, &P)))
         return rc;
-    cudaError_t e = launch_mixed_layer(P, grid_for(c, pl), st);
+    cudaError_t e = launch_mixed_layer(P, grid_for(c, pl), st, c->pdl);
     if (e != cudaSuccess)
         return cuda_fail(c, e, "mixed_layer launch");
     return MX_OK;
@@ -636,7 +637,7 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     if (timed && (e = cudaEventRecord(c->ev_start, st)) != cudaSuccess)
         return cuda_fail(c, e, "cudaEventRecord(start)");
     for (int l = 0; work && l < n_layers; ++l) {
-        e = launch_mixed_layer(params[l], grid_for(c, pl), st);
+        e = launch_mixed_layer(params[l], grid_for(c, pl), st, c->pdl);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "mixed_layer launch");
     }
@@ -688,6 +689,11 @@ int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
         if (value < 0 || value > 65535)
             return fail(c, MX_EINVAL, "prefill piece tiles must be in [0, 65535]");
         c->piece_tiles_opt = (int)value;
+        return MX_OK;
+    case MX_OPT_PDL:
+        if (value != 0 && value != 1)
+            return fail(c, MX_EINVAL, "MX_OPT_PDL is 0 or 1");
+        c->pdl = value != 0;
         return MX_OK;
     case MX_OPT_GRID:
         if (value < 0 || value > 65535)

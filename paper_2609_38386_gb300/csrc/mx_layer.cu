@@ -786,7 +786,6 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
             mbar_init(smem_u32(&misc->bar_odone[b]), 1);
         }
         misc->abort = 0;
-        misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
         fence_mbar_init();
         if (P.has_prefill) {
             tma_prefetch_desc(&P.tm_q);
@@ -800,6 +799,13 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         tmem_alloc(smem_u32(&misc->tmem_base), kTmemCols);
         tmem_relinquish();
     }
+    // The prologue above touches no global memory.  Let the next layer's grid
+    // launch onto SMs this grid frees, then wait for the previous layer (which
+    // shares the workspace: counters, partials) before the first fetch.
+    pdl_launch_dependents();
+    pdl_wait();
+    if (tid == 0)
+        misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -897,10 +903,19 @@ cudaError_t init_layer_kernel()
                                 kSmemTotal);
 }
 
-cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream)
+cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream, bool pdl)
 {
-    mixed_layer_kernel<<<grid, kThreads, kSmemTotal, stream>>>(P);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemTotal;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, mixed_layer_kernel, P);
 }
 
 cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int num_pages,

@@ -34,7 +34,7 @@
 
 namespace mx {
 cudaError_t init_layer_kernel();
-cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream);
+cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream, bool pdl);
 }  // namespace mx
 
 using namespace mx;
@@ -320,7 +320,7 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
                             cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess)
         return report(err_buf, err_len, MX_ECUDA, "staging the work list: %s", cudaGetErrorString(e));
-    e = launch_mixed_layer(P, std::max(1, std::min(st->num_sms, n)), s);
+    e = launch_mixed_layer(P, std::max(1, std::min(st->num_sms, n)), s, false);
     if (e != cudaSuccess)
         return report(err_buf, err_len, MX_ECUDA, "launch: %s", cudaGetErrorString(e));
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess)
