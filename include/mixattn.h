@@ -142,6 +142,8 @@ int mx_mixed_attention(mx_ctx *ctx, const mx_iter_desc *desc,
 
 /* A whole iteration: the same schedule `desc` run through n_layers layers
  * (layers[l] holds layer l's tensors), one launch per layer, planned once.
+ * The layers' tensors must be distinct (no layer reads what another writes):
+ * consecutive layer launches may overlap on the GPU (see MX_OPT_PDL).
  * With device_us_out != NULL: records CUDA events before the first and after
  * the last launch, waits for the second, and stores the elapsed device time in
  * microseconds in *device_us_out (the L_t of Eq. 1 as completed on the
@@ -168,9 +170,10 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
 #define MX_OPT_SPLIT_KEYS 1
 #define MX_OPT_GRID 2
 #define MX_OPT_PREFILL_PIECE_TILES 3
-/* MX_OPT_PDL: 1 (default) launches each layer kernel with programmatic
- * dependent launch, so the next layer's CTAs start their set-up on SMs the
- * previous layer has freed; 0 = ordinary stream order. */
+/* MX_OPT_PDL: 1 (default) launches layers 2..L of mx_iteration with
+ * programmatic dependent launch: a layer starts working on the SMs the
+ * previous layer frees once that layer's work queue has drained (consecutive
+ * launches use alternate workspace sets); 0 = ordinary stream order. */
 #define MX_OPT_PDL 4
 int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 

@@ -47,13 +47,17 @@ struct mx_ctx {
     int max_items = 0;
     // workspace (device)
     uint8_t *ws = nullptr;
-    float *part_o = nullptr;
-    float *part_lse = nullptr;
-    uint32_t *merge_cnt = nullptr;
-    float *pre_o = nullptr;
-    float *pre_lse = nullptr;
-    uint32_t *pre_cnt = nullptr;
-    uint32_t *work_cnt = nullptr;
+    // Two workspace sets, used by alternate launches: a layer kernel may
+    // start while the previous one drains (programmatic dependent launch),
+    // and the one before that has completed by then.
+    struct Set {
+        float *part_o, *part_lse;
+        uint32_t *merge_cnt;
+        float *pre_o, *pre_lse;
+        uint32_t *pre_cnt;
+        uint32_t *work_cnt;
+    } set[2] = {};
+    uint64_t launch_seq = 0;
     uint32_t *err = nullptr;
     uint8_t *plan_dev[kPlanSlots] = {};
     // pinned staging for the work list
@@ -325,7 +329,7 @@ int encode_map(mx_ctx *c, CUtensorMap *m, const void *base, int rank, const cuui
 }
 
 int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const Plan &pl,
-                LayerParams *P)
+                LayerParams *P, int set)
 {
     const mx_geom &g = c->g;
     std::memset(P, 0, sizeof *P);
@@ -340,13 +344,14 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->slots = d->slots;
     P->items = pl.items_dev;
     P->dec = pl.dec_dev;
-    P->part_o = c->part_o;
-    P->part_lse = c->part_lse;
-    P->merge_cnt = c->merge_cnt;
-    P->pre_o = c->pre_o;
-    P->pre_lse = c->pre_lse;
-    P->pre_cnt = c->pre_cnt;
-    P->work_cnt = c->work_cnt;
+    const mx_ctx::Set &w = c->set[set & 1];
+    P->part_o = w.part_o;
+    P->part_lse = w.part_lse;
+    P->merge_cnt = w.merge_cnt;
+    P->pre_o = w.pre_o;
+    P->pre_lse = w.pre_lse;
+    P->pre_cnt = w.pre_cnt;
+    P->work_cnt = w.work_cnt;
     P->err = c->err;
     P->n_items = pl.n_items;
     P->n_decodes = d->n_decodes;
@@ -489,26 +494,30 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     const size_t pre_cnt_bytes = (((size_t)max_qtiles * g->num_q_heads * sizeof(uint32_t)) + 255) & ~size_t(255);
     c->plan_bytes = plan_capacity_bytes(c);
     const size_t plan_stride = (c->plan_bytes + 255) & ~size_t(255);
-    const size_t total = part_o_bytes + part_lse_bytes + ((merge_bytes + 255) & ~size_t(255)) +
-                         pre_o_bytes + pre_lse_bytes + pre_cnt_bytes +
-                         256 /*counters + err*/ + kPlanSlots * plan_stride;
+    const size_t set_bytes = part_o_bytes + part_lse_bytes + ((merge_bytes + 255) & ~size_t(255)) +
+                             pre_o_bytes + pre_lse_bytes + pre_cnt_bytes + 256 /*work counters*/;
+    const size_t total = 2 * set_bytes + 256 /*error word*/ + kPlanSlots * plan_stride;
     if ((e = cudaMalloc(&c->ws, total)) != cudaSuccess)
         return bail(e, "cudaMalloc(workspace)");
     uint8_t *p = c->ws;
-    c->part_o = reinterpret_cast<float *>(p);
-    p += part_o_bytes;
-    c->part_lse = reinterpret_cast<float *>(p);
-    p += part_lse_bytes;
-    c->merge_cnt = reinterpret_cast<uint32_t *>(p);
-    p += (merge_bytes + 255) & ~size_t(255);
-    c->pre_o = reinterpret_cast<float *>(p);
-    p += pre_o_bytes;
-    c->pre_lse = reinterpret_cast<float *>(p);
-    p += pre_lse_bytes;
-    c->pre_cnt = reinterpret_cast<uint32_t *>(p);
-    p += pre_cnt_bytes;
-    c->work_cnt = reinterpret_cast<uint32_t *>(p);
-    c->err = c->work_cnt + 4;
+    for (int k = 0; k < 2; ++k) {
+        mx_ctx::Set &w = c->set[k];
+        w.part_o = reinterpret_cast<float *>(p);
+        p += part_o_bytes;
+        w.part_lse = reinterpret_cast<float *>(p);
+        p += part_lse_bytes;
+        w.merge_cnt = reinterpret_cast<uint32_t *>(p);
+        p += (merge_bytes + 255) & ~size_t(255);
+        w.pre_o = reinterpret_cast<float *>(p);
+        p += pre_o_bytes;
+        w.pre_lse = reinterpret_cast<float *>(p);
+        p += pre_lse_bytes;
+        w.pre_cnt = reinterpret_cast<uint32_t *>(p);
+        p += pre_cnt_bytes;
+        w.work_cnt = reinterpret_cast<uint32_t *>(p);
+        p += 256;
+    }
+    c->err = reinterpret_cast<uint32_t *>(p);
     p += 256;
     for (int s = 0; s < kPlanSlots; ++s) {
         c->plan_dev[s] = p;
@@ -518,10 +527,13 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
         if ((e = cudaEventCreateWithFlags(&c->plan_ev[s], cudaEventDisableTiming)) != cudaSuccess)
             return bail(e, "cudaEventCreate");
     }
-    if ((e = cudaMemset(c->merge_cnt, 0, merge_bytes)) != cudaSuccess ||
-        (e = cudaMemset(c->pre_cnt, 0, pre_cnt_bytes)) != cudaSuccess ||
-        (e = cudaMemset(c->work_cnt, 0, 256)) != cudaSuccess)
-        return bail(e, "cudaMemset(workspace)");
+    for (int k = 0; k < 2; ++k)
+        if ((e = cudaMemset(c->set[k].merge_cnt, 0, merge_bytes)) != cudaSuccess ||
+            (e = cudaMemset(c->set[k].pre_cnt, 0, pre_cnt_bytes)) != cudaSuccess ||
+            (e = cudaMemset(c->set[k].work_cnt, 0, 256)) != cudaSuccess)
+            return bail(e, "cudaMemset(workspace)");
+    if ((e = cudaMemset(c->err, 0, 256)) != cudaSuccess)
+        return bail(e, "cudaMemset(error word)");
     if ((e = cudaEventCreate(&c->ev_start)) != cudaSuccess ||
         (e = cudaEventCreate(&c->ev_end)) != cudaSuccess)
         return bail(e, "cudaEventCreate");
@@ -601,11 +613,13 @@ int mx_mixed_attention(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b,
     if ((rc = plan(c, d, st, &pl)))
         return rc;
     LayerParams P;
-    if ((rc = make_params(c, d, b, pl, &P)))
+    if ((rc = make_params(c, d, b, pl, &P, (int)(c->launch_seq & 1))))
         return rc;
-    cudaError_t e = launch_mixed_layer(P, grid_for(c, pl), st, c->pdl);
+    // ordinary stream order: the caller's next or previous work may depend on it
+    cudaError_t e = launch_mixed_layer(P, grid_for(c, pl), st, false);
     if (e != cudaSuccess)
         return cuda_fail(c, e, "mixed_layer launch");
+    ++c->launch_seq;
     return MX_OK;
 }
 
@@ -631,15 +645,19 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     // all descriptors are encoded before the timed region starts
     std::vector<LayerParams> params(work ? n_layers : 0);
     for (int l = 0; work && l < n_layers; ++l)
-        if ((rc = make_params(c, d, layers + l, pl, &params[l])))
+        if ((rc = make_params(c, d, layers + l, pl, &params[l], (int)((c->launch_seq + l) & 1))))
             return rc;
     cudaError_t e;
     if (timed && (e = cudaEventRecord(c->ev_start, st)) != cudaSuccess)
         return cuda_fail(c, e, "cudaEventRecord(start)");
+    // Layers of one iteration are independent (distinct tensors), so layer
+    // l > 0 may start while layer l - 1 drains; the first layer keeps
+    // ordinary stream order behind whatever the caller enqueued before.
     for (int l = 0; work && l < n_layers; ++l) {
-        e = launch_mixed_layer(params[l], grid_for(c, pl), st, c->pdl);
+        e = launch_mixed_layer(params[l], grid_for(c, pl), st, c->pdl && l > 0);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "mixed_layer launch");
+        ++c->launch_seq;
     }
     if (!timed)
         return MX_OK;

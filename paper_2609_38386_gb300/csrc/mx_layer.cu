@@ -799,11 +799,9 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         tmem_alloc(smem_u32(&misc->tmem_base), kTmemCols);
         tmem_relinquish();
     }
-    // The prologue above touches no global memory.  Let the next layer's grid
-    // launch onto SMs this grid frees, then wait for the previous layer (which
-    // shares the workspace: counters, partials) before the first fetch.
-    pdl_launch_dependents();
-    pdl_wait();
+    // Consecutive launches use alternate workspace sets, and the launch two
+    // back has completed before this one was launched (see the end of the
+    // kernel), so work starts at once, beside the previous layer's tail.
     if (tid == 0)
         misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
     tc_fence_before();
@@ -847,6 +845,12 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         buf ^= 1;
     }
 
+    // Out of work: once the previous launch has completed (it has, long ago),
+    // let the next launch start on the SMs this grid is freeing.  The next
+    // launch reuses the workspace set of the previous one, which is why this
+    // CTA waits for it first.
+    pdl_wait();
+    pdl_launch_dependents();
     if (misc->abort) {
         // give in-flight copies and MMAs time to land before TMEM is freed
         const uint64_t t0 = globaltimer_ns();
