@@ -128,6 +128,28 @@ def dist_setup():
     return ws, rank, local
 
 
+# Multi-GPU: independent replicas (the path partitions by request; no
+# exchange inside attention).  Each rank runs the whole workload on its own
+# GPU with its own seed; the job's time is the slowest rank's and its value
+# the tokens of all ranks over that time.
+def replica_seed_offset(rank: int) -> int:
+    return rank
+
+
+def max_over_ranks(value: float, ws: int, device=None) -> float:
+    if ws == 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_value(tokens_per_step: int, steps: int, ws: int, total_ms: float) -> float:
+    return tokens_per_step * steps * ws / (total_ms * 1e-3)
+
+
 # ------------------------------------------------------------ GPU workload
 class Workload:
     """Device-resident inputs of every iteration of a sweep, per layer."""
@@ -487,7 +509,7 @@ def main():
     peaks = load_peaks()
 
     layers = 2 if args.profile else None
-    w = Workload(cfg, device, seed_offset=rank, layers=layers)
+    w = Workload(cfg, device, seed_offset=replica_seed_offset(rank), layers=layers)
     if args.profile:
         keep = [i for i, it in enumerate(w.its) if it.chunk_size == args.profile_chunk][-2:]
         w.its = [w.its[i] for i in keep]
@@ -525,11 +547,7 @@ def main():
     clocks = sampler.stop()
     barrier()
     w.ctx.sync_status()
-    total_ms = t_start.elapsed_time(t_end)
-    if ws > 1:
-        t = torch.tensor([total_ms], device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), ws, device)
 
     it_us = np.array([[evs[s][i].elapsed_time(evs[s][i + 1]) * 1e3 for i in range(n_it)]
                       for s in range(args.steps)])          # [steps][iterations]
@@ -579,7 +597,7 @@ def main():
                                         / t_total),
                 "peak_source": peaks["source"], "kernel": "mixed_layer_kernel"}
 
-    value = w.tokens_per_step * args.steps * ws / (total_ms * 1e-3)
+    value = whole_job_value(w.tokens_per_step, args.steps, ws, total_ms)
     plan = w.ctx.last_plan()
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
