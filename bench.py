@@ -154,7 +154,7 @@ def whole_job_value(tokens_per_step: int, steps: int, ws: int, total_ms: float) 
 class Workload:
     """Device-resident inputs of every iteration of a sweep, per layer."""
 
-    def __init__(self, cfg, device, seed_offset=0, layers=None):
+    def __init__(self, cfg, device, seed_offset=0, layers=None, lean=False):
         import torch
 
         import synth
@@ -184,17 +184,36 @@ class Workload:
         self.outs = [torch.empty((self.max_tok, g.hq, g.head_dim), dtype=torch.int16,
                                  device=device) for _ in range(self.L)]
         self.descs, self.layer_arrays, self.inputs, self.slots = [], [], [], []
+        shared = []
+        if lean:
+            # one q/k/v buffer per layer, sized for the largest iteration and
+            # reused by every iteration: for sweeps whose per-iteration inputs
+            # do not fit (the 32B sweep would need ~225 GB of them)
+            big = max(self.its, key=lambda it: it.n_tokens)
+            for l in range(self.L):
+                q = torch.empty((self.max_tok, g.hq, g.head_dim), dtype=torch.int16, device=device)
+                k = torch.empty((self.max_tok, g.hkv, g.head_dim), dtype=torch.int16, device=device)
+                v = torch.empty_like(k)
+                sdev.fill_tokens_(q, self.seed, l, synth.STREAM_Q, big)
+                sdev.fill_tokens_(k, self.seed, l, synth.STREAM_K, big)
+                sdev.fill_tokens_(v, self.seed, l, synth.STREAM_V, big)
+                shared.append((q, k, v))
         for it in self.its:
             sl = torch.from_numpy(it.slots(lay)).to(device)
             self.slots.append(sl)
             bufs, keep = [], []
             for l in range(self.L):
-                q = torch.empty((it.n_tokens, g.hq, g.head_dim), dtype=torch.int16, device=device)
-                k = torch.empty((it.n_tokens, g.hkv, g.head_dim), dtype=torch.int16, device=device)
-                v = torch.empty_like(k)
-                sdev.fill_tokens_(q, self.seed, l, synth.STREAM_Q, it)
-                sdev.fill_tokens_(k, self.seed, l, synth.STREAM_K, it)
-                sdev.fill_tokens_(v, self.seed, l, synth.STREAM_V, it)
+                if lean:
+                    q, k, v = shared[l]
+                else:
+                    q = torch.empty((it.n_tokens, g.hq, g.head_dim), dtype=torch.int16,
+                                    device=device)
+                    k = torch.empty((it.n_tokens, g.hkv, g.head_dim), dtype=torch.int16,
+                                    device=device)
+                    v = torch.empty_like(k)
+                    sdev.fill_tokens_(q, self.seed, l, synth.STREAM_Q, it)
+                    sdev.fill_tokens_(k, self.seed, l, synth.STREAM_K, it)
+                    sdev.fill_tokens_(v, self.seed, l, synth.STREAM_V, it)
                 keep.append((q, k, v))
                 kp, vp = self.pools[l]
                 bufs.append(self.ctx.make_bufs(q, k, v, kp, vp, self.outs[l]))
@@ -451,6 +470,8 @@ def main():
     ap.add_argument("--profile-chunk", type=int, default=2048)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--lean", action="store_true",
+                    help="one q/k/v buffer per layer reused by all iterations (large sweeps)")
     ap.add_argument("--workload", default="sweep", choices=["sweep", "trace"],
                     help="trace: the completion-timed DLFP loop vs a fixed chunk cap")
     args = ap.parse_args()
@@ -463,8 +484,9 @@ def main():
               "decode_ctx": f"{cfg.ctx_dist}[{cfg.ctx_lo},{cfg.ctx_hi}]",
               "prompt_len": cfg.prompt_len, "chunk_sizes": list(cfg.chunk_sizes),
               "iterations_per_step": len(cfg.iterations()),
-              "l2": "inputs larger than L2: each iteration reads 28 distinct ~335 MB "
-                    "per-layer pools", "parallelism": f"replicas{ws}"}
+              "l2": f"inputs larger than L2: each iteration reads {cfg.n_layers} distinct "
+                    "per-layer KV pools of several hundred MB or more",
+              "parallelism": f"replicas{ws}"}
 
     if args.impl == "reference":
         if rank != 0:
@@ -509,7 +531,10 @@ def main():
     peaks = load_peaks()
 
     layers = 2 if args.profile else None
-    w = Workload(cfg, device, seed_offset=replica_seed_offset(rank), layers=layers)
+    w = Workload(cfg, device, seed_offset=replica_seed_offset(rank), layers=layers,
+                 lean=args.lean)
+    if args.lean:
+        config["inputs"] = "one q/k/v buffer per layer, reused by every iteration"
     if args.profile:
         keep = [i for i, it in enumerate(w.its) if it.chunk_size == args.profile_chunk][-2:]
         w.its = [w.its[i] for i in keep]

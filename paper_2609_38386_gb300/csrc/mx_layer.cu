@@ -341,6 +341,24 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
         P.merge_cnt[di * P.hkv + h] = 0u;
 }
 
+// Keys [r0, end of r0's page) of the last cached tile are not cached yet (the
+// chunk's own keys start there): zero their value rows in the staged V tile
+// so that P.V adds nothing for them (later pages were zero-filled by TMA).
+__device__ __forceinline__ void clear_uncached_rows(uint32_t dv, int r0)
+{
+    const int r1 = min(kTileN, (r0 + kPage - 1) / kPage * kPage);
+#pragma unroll 1
+    for (int r = r0; r < r1; ++r)
+#pragma unroll 1
+        for (int hf = 0; hf < 2; ++hf)
+#pragma unroll 1
+            for (int cc = 0; cc < 8; ++cc)
+                asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(dv + hf * kHalfTile + r * 128 + cc * 16),
+                             "r"(0u)
+                             : "memory");
+    fence_proxy_async_smem();
+}
+
 // ---------------------------------------------------------------------------
 // Prefill tile: rows [128t, 128t + 128) of the chunk, query head hq.
 // Key tiles: nA paged tiles covering [0, chunk_start), then t + 1 tiles of
@@ -434,66 +452,56 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
+        // One straight loop: S_i = Q K_i^T is issued before P_{i-1} V_{i-1},
+        // so the softmax of tile i overlaps the P.V of tile i - 1.  The
+        // descriptors are formed once per tile and advanced by constants.
         if (lane == 0) {
             bool ok = mbar_wait(bar_q, item_no & 1, abort, tmo);
             tc_fence_after();
-            auto issue_pv = [&](int i) -> bool {
-                const uint32_t c = tile0 + i;
-                const int st = c % kVStages;
-                const uint32_t ph = (c / kVStages) & 1;
-                if (!mbar_wait(smem_u32(&misc->bar_pfull[c & 1]), (c >> 1) & 1, abort, tmo))
-                    return false;
-                if (!mbar_wait(smem_u32(&misc->bar_vfull[st]), ph, abort, tmo))
-                    return false;
-                const uint32_t dv = sV + st * kTileBytes;
-                if (kt0 + i == nA - 1 && (cs % kTileN) != 0) {
-                    // keys [cs, end of that page) of the last paged tile are not
-                    // cached yet: clear their value rows (later pages are zero).
-                    const int r0 = cs - (kt0 + i) * kTileN;
-                    const int r1 = min(kTileN, (r0 + kPage - 1) / kPage * kPage);
-                    for (int r = r0; r < r1; ++r)
-                        for (int hf = 0; hf < 2; ++hf)
-                            for (int cc = 0; cc < 8; ++cc)
-                                asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(
-                                                 dv + hf * kHalfTile + r * 128 + cc * 16),
-                                             "r"(0u)
-                                             : "memory");
-                    fence_proxy_async_smem();
-                }
-                tc_fence_after();
-                const uint32_t pa = tmem + kTmemP + (c & 1) * 64;  // P_c: 8 columns per 16 keys
+            for (int i = 0; ok && i <= nT; ++i) {
+                if (i < nT) {
+                    const uint32_t c = tile0 + i;
+                    const int st = c % kKStages;
+                    if (!mbar_wait(smem_u32(&misc->bar_kfull[st]), (c / kKStages) & 1, abort, tmo)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t qdesc = smem_desc(sQ, 16, 1024, kSwz128);
+                    const uint64_t kdesc = smem_desc(sK + st * kTileBytes, 16, 1024, kSwz128);
+                    const uint32_t d = tmem + (c & 1) * 128;
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const uint64_t b = smem_desc(dv + kk * 2048, kHalfTile, 1024, kSwz128);
-                    tc_mma_ts(tmem + kTmemO, pa + kk * 8, b, kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
+                    for (int kk = 0; kk < 8; ++kk) {
+                        // 16 keys of K-major SW128: +32 B inside a 64-column half
+                        const uint64_t off = (uint64_t)(((kk >> 2) * kHalfTile + (kk & 3) * 32) >> 4);
+                        tc_mma_ss(d, qdesc + off, kdesc + off, kIdescS, kk > 0 ? 1u : 0u);
+                    }
+                    tc_commit(smem_u32(&misc->bar_sfull[c & 1]));
+                    tc_commit(smem_u32(&misc->bar_kempty[st]));
                 }
-                tc_commit(smem_u32(&misc->bar_odone[c & 1]));
-                tc_commit(smem_u32(&misc->bar_vempty[st]));
-                return true;
-            };
-            for (int i = 0; ok && i < nT; ++i) {
-                const uint32_t c = tile0 + i;
-                const int st = c % kKStages;
-                const uint32_t ph = (c / kKStages) & 1;
-                if (!mbar_wait(smem_u32(&misc->bar_kfull[st]), ph, abort, tmo)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t dk = sK + st * kTileBytes;
+                if (i > 0) {
+                    const int j = i - 1;
+                    const uint32_t c = tile0 + j;
+                    const int st = c % kVStages;
+                    if (!mbar_wait(smem_u32(&misc->bar_pfull[c & 1]), (c >> 1) & 1, abort, tmo) ||
+                        !mbar_wait(smem_u32(&misc->bar_vfull[st]), (c / kVStages) & 1, abort, tmo)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t dv = sV + st * kTileBytes;
+                    if (kt0 + j == nA - 1 && (cs % kTileN) != 0)
+                        clear_uncached_rows(dv, cs - (kt0 + j) * kTileN);
+                    tc_fence_after();
+                    const uint64_t vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
+                    const uint32_t pa = tmem + kTmemP + (c & 1) * 64;  // P_c: 8 columns per 16 keys
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const uint64_t a = smem_desc(sQ + (kk >> 2) * kHalfTile + (kk & 3) * 32, 16, 1024, kSwz128);
-                    const uint64_t b = smem_desc(dk + (kk >> 2) * kHalfTile + (kk & 3) * 32, 16, 1024, kSwz128);
-                    tc_mma_ss(tmem + (c & 1) * 128, a, b, kIdescS, kk > 0 ? 1u : 0u);
+                    for (int kk = 0; kk < 8; ++kk)  // 16 keys of MN-major V: +2 KiB
+                        tc_mma_ts(tmem + kTmemO, pa + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4), kIdescO,
+                                  (j > 0 || kk > 0) ? 1u : 0u);
+                    tc_commit(smem_u32(&misc->bar_odone[c & 1]));
+                    tc_commit(smem_u32(&misc->bar_vempty[st]));
                 }
-                tc_commit(smem_u32(&misc->bar_sfull[c & 1]));
-                tc_commit(smem_u32(&misc->bar_kempty[st]));
-                if (i > 0 && !issue_pv(i - 1))
-                    ok = false;
             }
-            if (ok && !issue_pv(nT - 1))
-                ok = false;
             if (!ok)
                 set_abort(P, misc);
         }
@@ -562,7 +570,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             const int nvalid = gi < nA ? min(kTileN, cs - gi * kTileN)
                                        : min(kTileN, j - kTileN * (gi - nA) + 1);
             // Pass 1: row max of the raw scores (the scale is positive) over
-            // the two 64-column halves of S, 8 independent chains.  S is read
+            // the two 64-column halves of S, 8 independent three-input chains.  S is read
             // from TMEM twice (here and in pass 2) to keep only 64 scores live.
             float mx8[8];
 #pragma unroll
@@ -581,8 +589,8 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                             sv[cc] = 0xFF800000u;
                 }
 #pragma unroll
-                for (int cc = 0; cc < 64; ++cc)
-                    mx8[cc & 7] = fmaxf(mx8[cc & 7], __uint_as_float(sv[cc]));
+                for (int cc = 0; cc < 32; ++cc)
+                    mx8[cc & 7] = max3(mx8[cc & 7], __uint_as_float(sv[2 * cc]), __uint_as_float(sv[2 * cc + 1]));
             }
             const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                                    fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
@@ -617,7 +625,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 l_run *= alpha;
             }
             // Pass 2: p = 2^(s*scale - m) as bf16 pairs into TMEM lane r (the A
-            // operand of P.V), and the row sum with 8 chains.
+            // operand of P.V), and the row sum in 4 packed pair chains.
             float rs8[8];
 #pragma unroll
             for (int u = 0; u < 8; ++u)
@@ -637,9 +645,10 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 uint32_t pk[32];
 #pragma unroll
                 for (int cc = 0; cc < 32; ++cc) {
-                    const float e0 = ex2(fmaf(__uint_as_float(sv[2 * cc]), sl, nm));
-                    const float e1 = ex2(fmaf(__uint_as_float(sv[2 * cc + 1]), sl, nm));
-                    rs8[cc & 7] += e0 + e1;
+                    float x0, x1;
+                    ffma2(x0, x1, __uint_as_float(sv[2 * cc]), __uint_as_float(sv[2 * cc + 1]), sl, sl, nm, nm);
+                    const float e0 = ex2(x0), e1 = ex2(x1);
+                    fadd2(rs8[2 * (cc & 3)], rs8[2 * (cc & 3) + 1], e0, e1);
                     pk[cc] = pack_bf16(e0, e1);
                 }
                 tmem_st32(tl + kTmemP + (c & 1) * 64 + 32 * half, pk);
