@@ -55,12 +55,28 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
     return ok != 0;
 }
 
+// Non-blocking probe of the same phase.  Issued right after queued
+// tcgen05.mma instructions it returns sooner than try_wait, which the
+// MMA-issuing thread pays for at every wait between MMA groups.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait: returns false after `limit_ns` of wall time (globaltimer) or
 // as soon as *abort becomes nonzero.  Never spins forever.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
                                           volatile int *abort, uint64_t limit_ns)
 {
-    if (mbar_try_wait(bar, parity))
+    if (mbar_test_wait(bar, parity))
         return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t it = 1;; ++it) {
