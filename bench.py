@@ -420,9 +420,11 @@ class TraceEngine:
 
 
 def trace_measure(device, seeds=(801, 802, 803), n_layers=28, hq=16, budget=8192,
-                  max_seqs=64, fixed_cap=2048):
-    """Config 5: the completion-timed DLFP loop against a fixed chunk cap on
-    seeded open-loop traces (§3.1 Eq. 2 with L_t = device-completion time)."""
+                  max_seqs=64, fixed_caps=(2048, 3072, 4096), loads=(20.0, 5.0)):
+    """Config 5: the completion-timed DLFP loop against fixed chunk caps on
+    seeded open-loop traces (§3.1 Eq. 2 with L_t = device-completion time).
+    `loads` are mean inter-arrival times in units of t_ref (20 is the
+    reference load; smaller is heavier)."""
     import numpy as np
     import torch
 
@@ -436,24 +438,29 @@ def trace_measure(device, seeds=(801, 802, 803), n_layers=28, hq=16, budget=8192
     t_ref = float(np.median([eng.execute(cal) for _ in range(7)]))
     del eng
     torch.cuda.empty_cache()
-    result = {"t_ref_us": t_ref, "mean_interarrival_us": 20 * t_ref, "target_us": t_ref,
-              "fixed_cap": fixed_cap, "seeds": {}}
-    red = []
-    for seed in seeds:
-        spec = dlfp.TraceSpec(mean_interarrival=20 * t_ref, seed=seed)
-        eng = TraceEngine(spec.requests(), n_layers, hq, device, seed, budget, max_seqs)
-        per = {}
-        for name in ("fixed", "dlfp"):
-            ctl = dlfp.FixedCap(fixed_cap) if name == "fixed" else dlfp.DLFPController(t_ref)
-            sch = dlfp.Scheduler(spec.requests(), ctl, max_seqs=max_seqs, budget=budget)
-            t0 = time.perf_counter()
-            per[name] = sch.run(eng.execute)
-            per[name]["wall_s"] = time.perf_counter() - t0
-        red.append(1 - per["dlfp"]["itl_p99"] / per["fixed"]["itl_p99"])
-        result["seeds"][str(seed)] = per
-        del eng
-        torch.cuda.empty_cache()
-    result["mean_itl_p99_reduction"] = float(np.mean(red))
+    result = {"t_ref_us": t_ref, "target_us": t_ref, "fixed_caps": list(fixed_caps), "loads": {}}
+    policies = [f"fixed{c}" for c in fixed_caps] + ["dlfp"]
+    for load in loads:
+        per_load = {"mean_interarrival_us": load * t_ref, "seeds": {}}
+        red = {f"fixed{c}": [] for c in fixed_caps}
+        for seed in seeds:
+            spec = dlfp.TraceSpec(mean_interarrival=load * t_ref, seed=seed)
+            eng = TraceEngine(spec.requests(), n_layers, hq, device, seed, budget, max_seqs)
+            per = {}
+            for name in policies:
+                ctl = (dlfp.DLFPController(t_ref) if name == "dlfp"
+                       else dlfp.FixedCap(int(name[len("fixed"):])))
+                sch = dlfp.Scheduler(spec.requests(), ctl, max_seqs=max_seqs, budget=budget)
+                t0 = time.perf_counter()
+                per[name] = sch.run(eng.execute)
+                per[name]["wall_s"] = time.perf_counter() - t0
+            for c in fixed_caps:
+                red[f"fixed{c}"].append(1 - per["dlfp"]["itl_p99"] / per[f"fixed{c}"]["itl_p99"])
+            per_load["seeds"][str(seed)] = per
+            del eng
+            torch.cuda.empty_cache()
+        per_load["mean_itl_p99_reduction_vs"] = {k: float(np.mean(v)) for k, v in red.items()}
+        result["loads"][f"{load:g}"] = per_load
     return result
 
 
@@ -519,7 +526,7 @@ def main():
             torch.cuda.set_device(device)
             res = trace_measure(device)
             print(json.dumps({"metric": "open-loop trace: per-iteration device us P50/P99 and "
-                              "ITL/TTFT, completion-timed DLFP vs fixed chunk cap",
+                              "ITL/TTFT, completion-timed DLFP vs fixed chunk caps",
                               "workload": "qwen3-0.6b-attn-28L-poisson-trace", **res}))
         return
     if ws > 1:
