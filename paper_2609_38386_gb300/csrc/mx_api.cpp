@@ -181,7 +181,10 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
 
     int split = c->split_keys_opt;
     if (split <= 0) {
-        const int64_t target_items = 2LL * c->num_sms;
+        // Each split pays a fixed start-up and merge cost, so splits are as long
+        // as load balance allows: about 1.5 per SM for a decode-only iteration,
+        // one per SM beside prefill tiles (which fill the rest of the launch).
+        const int64_t target_items = d->p_t > 0 ? (int64_t)c->num_sms : 3LL * c->num_sms / 2;
         int64_t s = (total_keys + target_items - 1) / std::max<int64_t>(target_items, 1);
         s = (s + 127) / 128 * 128;
         split = (int)std::min<int64_t>(std::max<int64_t>(s, 512), kMaxSplitKeys);
