@@ -34,16 +34,16 @@ struct Misc {
     uint64_t bar_kfull[kKStages];
     uint64_t bar_kempty[kKStages];
     uint64_t bar_vfull[kVStages];
-    uint64_t bar_vempty[kVStages];
     uint64_t bar_sfull[2];
     uint64_t bar_pfull[2];
-    uint64_t bar_odone[2];
+    uint64_t bar_odone[2];  // P.V of P buffer b done; frees P buffer b and V stage b
     uint32_t tmem_base;
     int32_t item_idx[2];
     int32_t abort;
     int32_t last;
 };
 static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
+static_assert(kVStages == 2, "V stage c % 2 is released by the odone barrier of P buffer c & 1");
 
 // Instruction descriptors: S = Q K^T (both K-major) and O = P V (V MN-major).
 constexpr uint32_t kIdescS = idesc_bf16_f32(128, 128, false, false);
@@ -395,7 +395,9 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
         const void *tm_in = isK ? (const void *)&P.tm_k : (const void *)&P.tm_v;
         uint64_t *full = isK ? misc->bar_kfull : misc->bar_vfull;
-        uint64_t *empty = isK ? misc->bar_kempty : misc->bar_vempty;
+        // V stage c % 2 is free once P_{c-2} V_{c-2} has completed, which is
+        // exactly the odone barrier of P buffer c & 1 (one commit fewer per tile).
+        uint64_t *empty = isK ? misc->bar_kempty : misc->bar_odone;
         const int oob_row = P.num_pages * P.hkv * kPage;
         for (int i = 0; i < nT; ++i) {
             const uint32_t c = tile0 + i;
@@ -455,6 +457,9 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         // One straight loop: S_i = Q K_i^T is issued before P_{i-1} V_{i-1},
         // so the softmax of tile i overlaps the P.V of tile i - 1.  The
         // descriptors are formed once per tile and advanced by constants.
+        // A wait issued behind queued MMAs returns only once they have been
+        // accepted (the tensor pipe drains and refills), so each MMA group
+        // costs one such boundary and the commits are kept to a minimum.
         if (lane == 0) {
             bool ok = mbar_wait(bar_q, item_no & 1, abort, tmo);
             tc_fence_after();
@@ -498,8 +503,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                     for (int kk = 0; kk < 8; ++kk)  // 16 keys of MN-major V: +2 KiB
                         tc_mma_ts(tmem + kTmemO, pa + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4), kIdescO,
                                   (j > 0 || kk > 0) ? 1u : 0u);
-                    tc_commit(smem_u32(&misc->bar_odone[c & 1]));
-                    tc_commit(smem_u32(&misc->bar_vempty[st]));
+                    tc_commit(smem_u32(&misc->bar_odone[c & 1]));  // also frees V stage st
                 }
             }
             if (!ok)
@@ -787,7 +791,6 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         }
         for (int b = 0; b < kVStages; ++b) {
             mbar_init(smem_u32(&misc->bar_vfull[b]), 1);
-            mbar_init(smem_u32(&misc->bar_vempty[b]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&misc->bar_sfull[b]), 1);
