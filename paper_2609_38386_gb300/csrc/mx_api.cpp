@@ -34,7 +34,7 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
 constexpr int kPlanSlots = 4;         // ring of work-list buffers
 constexpr int kPartSlots = 16384;     // decode split partials capacity
 constexpr int kPrePartSlots = 1024;   // prefill piece partials capacity (64 KiB each)
-constexpr int kMinPieceTiles = 32;    // smallest prefill piece, in 128-key tiles
+constexpr int kMinPieceTiles = 48;    // smallest prefill piece, in 128-key tiles
 constexpr int kMaxSplitKeys = kWarps * 32 * kPage;  // 4096: one page id per lane
 constexpr uint64_t kTimeoutNs = 1000000000ull;      // 1 s bound on in-kernel waits
 
@@ -227,7 +227,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         pre_work += (int64_t)(nA + t + 1) * hq;
     // Splitting costs a partial write and a merge; it pays only when the
     // chunk has too few tiles to occupy the GPU (short chunks deep into a
-    // long prompt), so tiles are split only then, into >= 32-tile pieces.
+    // long prompt), so tiles are split only then, into >= 48-tile pieces.
     int piece = c->piece_tiles_opt;
     if (piece <= 0) {
         if ((int64_t)n_qt * hq * 2 >= c->num_sms)
