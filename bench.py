@@ -238,9 +238,14 @@ class Workload:
 
 
 def e2e_measure(w, steps, device):
-    """Same sweep through the iteration call with host buffers: per iteration,
-    copy every layer's q/k/v from pinned host memory, run the iteration and
-    wait for its completion time, copy every layer's output back."""
+    """Same sweep through the iteration call with host buffers: every
+    iteration's q/k/v for all layers is copied from pinned host memory, the
+    iteration runs, and every layer's output is copied back to pinned host
+    memory, all inside the timed region.  The copies are pipelined against the
+    iterations the way a serving loop would run them: the inputs of iteration
+    i+1 and i+2 upload on one stream and the outputs of iteration i-1
+    download on another while iteration i computes (three device buffer
+    sets, so that a large iteration's upload has two iterations of slack)."""
     import torch
     g, L = w.geom, w.L
     per_tok_in = (g.hq + 2 * g.hkv) * g.head_dim
@@ -249,8 +254,9 @@ def e2e_measure(w, steps, device):
     max_out = L * w.max_tok * per_tok_out
     h_in = torch.empty(max_in, dtype=torch.int16, pin_memory=True)
     h_out = torch.empty(max_out, dtype=torch.int16, pin_memory=True)
-    d_in = torch.empty(max_in, dtype=torch.int16, device=device)
-    d_out = torch.empty(max_out, dtype=torch.int16, device=device)
+    nbuf = 3
+    d_in = [torch.empty(max_in, dtype=torch.int16, device=device) for _ in range(nbuf)]
+    d_out = [torch.empty(max_out, dtype=torch.int16, device=device) for _ in range(nbuf)]
     # host contents: the largest iteration's device inputs, packed per layer
     big = max(range(len(w.its)), key=lambda i: w.its[i].n_tokens)
     off = 0
@@ -259,47 +265,67 @@ def e2e_measure(w, steps, device):
             n = t.numel()
             h_in[off:off + n].copy_(t.reshape(-1).cpu())
             off += n
-    layer_arrays, in_bytes, out_bytes = [], [], []
+    layer_arrays, in_elems, out_elems = [], [], []
     for i, it in enumerate(w.its):
         n = it.n_tokens
-        bufs, o_in, o_out = [], 0, 0
-        for l in range(L):
-            q = d_in[o_in:o_in + n * g.hq * g.head_dim]
-            o_in += q.numel()
-            k = d_in[o_in:o_in + n * g.hkv * g.head_dim]
-            o_in += k.numel()
-            v = d_in[o_in:o_in + n * g.hkv * g.head_dim]
-            o_in += v.numel()
-            out = d_out[o_out:o_out + n * per_tok_out]
-            o_out += out.numel()
-            kp, vp = w.pools[l]
-            bufs.append(w.ctx.make_bufs(q, k, v, kp, vp, out))
-        layer_arrays.append(w.ctx.layer_array(bufs))
-        in_bytes.append(o_in * 2)
-        out_bytes.append(o_out * 2)
-    stream = torch.cuda.current_stream(device)
+        sets = []
+        for b in range(nbuf):
+            bufs, o_in, o_out = [], 0, 0
+            for l in range(L):
+                q = d_in[b][o_in:o_in + n * g.hq * g.head_dim]
+                o_in += q.numel()
+                k = d_in[b][o_in:o_in + n * g.hkv * g.head_dim]
+                o_in += k.numel()
+                v = d_in[b][o_in:o_in + n * g.hkv * g.head_dim]
+                o_in += v.numel()
+                out = d_out[b][o_out:o_out + n * per_tok_out]
+                o_out += out.numel()
+                kp, vp = w.pools[l]
+                bufs.append(w.ctx.make_bufs(q, k, v, kp, vp, out))
+            sets.append(w.ctx.layer_array(bufs))
+        layer_arrays.append(sets)
+        in_elems.append(o_in)
+        out_elems.append(o_out)
+    comp = torch.cuda.current_stream(device)
+    up = torch.cuda.Stream(device)
+    down = torch.cuda.Stream(device)
+    n_it = len(w.its)
 
     def one_step():
-        dev_us = []
-        for i in range(len(w.its)):
-            ni, no = in_bytes[i] // 2, out_bytes[i] // 2
-            d_in[:ni].copy_(h_in[:ni], non_blocking=True)
-            dev_us.append(w.ctx.iteration(w.descs[i], layer_arrays[i], stream=stream, wait=True))
-            h_out[:no].copy_(d_out[:no], non_blocking=True)
-            stream.synchronize()
-        return dev_us
+        ev_in = [torch.cuda.Event() for _ in range(n_it)]
+        ev_comp = [torch.cuda.Event() for _ in range(n_it)]
+        ev_out = [torch.cuda.Event() for _ in range(n_it)]
+        for i in range(n_it):
+            b = i % nbuf
+            with torch.cuda.stream(up):
+                if i >= nbuf:
+                    up.wait_event(ev_comp[i - nbuf])   # inputs of i-nbuf consumed
+                d_in[b][:in_elems[i]].copy_(h_in[:in_elems[i]], non_blocking=True)
+                ev_in[i].record(up)
+            comp.wait_event(ev_in[i])
+            if i >= nbuf:
+                comp.wait_event(ev_out[i - nbuf])      # outputs of i-nbuf downloaded
+            w.ctx.iteration(w.descs[i], layer_arrays[i][b], stream=comp, wait=False)
+            ev_comp[i].record(comp)
+            with torch.cuda.stream(down):
+                down.wait_event(ev_comp[i])
+                h_out[:out_elems[i]].copy_(d_out[b][:out_elems[i]], non_blocking=True)
+                ev_out[i].record(down)
+        for s_ in (up, comp, down):
+            s_.synchronize()
 
     one_step()  # warm-up
+    w.ctx.sync_status()
     torch.cuda.synchronize(device)
     t0 = time.perf_counter()
-    all_us = []
     for _ in range(steps):
-        all_us += one_step()
+        one_step()
     torch.cuda.synchronize(device)
     dt = time.perf_counter() - t0
+    w.ctx.sync_status()
     return {"value": w.tokens_per_step * steps / dt, "unit": UNIT,
-            "h2d_bytes_per_step": int(sum(in_bytes)), "d2h_bytes_per_step": int(sum(out_bytes)),
-            "seconds": dt, "iteration_device_us_median": float(np.median(all_us))}
+            "h2d_bytes_per_step": int(sum(in_elems) * 2), "d2h_bytes_per_step": int(sum(out_elems) * 2),
+            "seconds": dt, "copies": "pinned host <-> device, overlapped with compute on two copy streams"}
 
 
 # ------------------------------------------------------------- CPU oracle
@@ -636,7 +662,8 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded N(0,1) bf16, random page permutation)",
             "config": config, "roofline": roofline, "per_chunk": per_chunk,
-            "gpu_launches": L * n_it * args.steps, "clocks": clocks,
+            # per iteration: one plan-upload kernel and one mixed_layer_kernel per layer
+            "gpu_launches": (L + 1) * n_it * args.steps, "clocks": clocks,
             "plan_last": plan}
     if not args.no_e2e and not args.profile:
         line["e2e"] = e2e_measure(w, max(1, min(args.steps, 3)), device)

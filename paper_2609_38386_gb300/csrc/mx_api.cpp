@@ -17,6 +17,7 @@
 namespace mx {
 cudaError_t init_layer_kernel();
 cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream, bool pdl);
+cudaError_t launch_plan_upload(const void *src, void *dst, size_t bytes, cudaStream_t stream);
 cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int num_pages,
                              const uint16_t *k, const uint16_t *v, uint16_t *k_pool,
                              uint16_t *v_pool, uint32_t *err, cudaStream_t stream);
@@ -62,6 +63,7 @@ struct mx_ctx {
     uint8_t *plan_dev[kPlanSlots] = {};
     // pinned staging for the work list
     uint8_t *plan_host[kPlanSlots] = {};
+    const void *plan_host_dev[kPlanSlots] = {};  // device view of plan_host (mapped pinned memory)
     cudaEvent_t plan_ev[kPlanSlots] = {};
     bool plan_ev_used[kPlanSlots] = {};
     size_t plan_bytes = 0;
@@ -297,9 +299,12 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         items[n++] = decode_item_code(x.i, x.h, x.s);
 
     const size_t bytes = items_off + (size_t)n * sizeof(int4);
-    cudaError_t e = cudaMemcpyAsync(c->plan_dev[slot], host, bytes, cudaMemcpyHostToDevice, stream);
+    // A kernel, not a copy engine, moves the plan: an H2D memcpy on the
+    // caller's stream would queue behind the caller's own large uploads (one
+    // copy engine per direction serves all streams in order).
+    cudaError_t e = launch_plan_upload(c->plan_host_dev[slot], c->plan_dev[slot], bytes, stream);
     if (e != cudaSuccess)
-        return cuda_fail(c, e, "cudaMemcpyAsync(plan)");
+        return cuda_fail(c, e, "plan upload");
     e = cudaEventRecord(c->plan_ev[slot], stream);
     if (e != cudaSuccess)
         return cuda_fail(c, e, "cudaEventRecord(plan)");
@@ -527,6 +532,10 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
         p += plan_stride;
         if ((e = cudaMallocHost(&c->plan_host[s], c->plan_bytes)) != cudaSuccess)
             return bail(e, "cudaMallocHost(plan)");
+        void *dv = nullptr;
+        if ((e = cudaHostGetDevicePointer(&dv, c->plan_host[s], 0)) != cudaSuccess)
+            return bail(e, "cudaHostGetDevicePointer(plan)");
+        c->plan_host_dev[s] = dv;
         if ((e = cudaEventCreateWithFlags(&c->plan_ev[s], cudaEventDisableTiming)) != cudaSuccess)
             return bail(e, "cudaEventCreate");
     }

@@ -934,6 +934,24 @@ cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stre
     return cudaLaunchKernelEx(&cfg, mixed_layer_kernel, P);
 }
 
+// Plan upload: the work list and decode table, read by the GPU from mapped
+// pinned host memory (16-byte words).
+__global__ void plan_upload_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst, int n)
+{
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+        dst[i] = src[i];
+}
+
+cudaError_t launch_plan_upload(const void *src, void *dst, size_t bytes, cudaStream_t stream)
+{
+    const int n = (int)(bytes / sizeof(uint4));
+    if (n == 0)
+        return cudaSuccess;
+    const int blocks = n < 8 * 256 ? (n + 255) / 256 : 8;
+    plan_upload_kernel<<<blocks, 256, 0, stream>>>(static_cast<const uint4 *>(src), static_cast<uint4 *>(dst), n);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int num_pages,
                              const uint16_t *k, const uint16_t *v, uint16_t *k_pool,
                              uint16_t *v_pool, uint32_t *err, cudaStream_t stream)
