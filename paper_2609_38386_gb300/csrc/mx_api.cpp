@@ -296,7 +296,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     std::stable_sort(ditems.begin(), ditems.end(),
                      [](const DItem &a, const DItem &b) { return a.keys > b.keys; });
     for (const DItem &x : ditems)
-        items[n++] = decode_item_code(x.i, x.h, x.s);
+        items[n++] = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx);
 
     const size_t bytes = items_off + (size_t)n * sizeof(int4);
     // A kernel, not a copy engine, moves the plan: an H2D memcpy on the
@@ -459,7 +459,7 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     if (!out || !g)
         return MX_EINVAL;
     *out = nullptr;
-    if (g->head_dim != kHeadDim || g->page_size != kPage || g->num_kv_heads <= 0 ||
+    if (g->head_dim != kHeadDim || g->page_size != kPage || g->num_kv_heads <= 0 || g->num_kv_heads > 255 ||
         g->num_q_heads <= 0 || g->num_q_heads % g->num_kv_heads != 0 ||
         g->num_q_heads / g->num_kv_heads > kMaxRep || g->num_pages <= 0 || g->num_seqs <= 0 ||
         g->max_pages_per_seq <= 0 || g->max_tokens < 0 || g->max_decodes < 0 ||

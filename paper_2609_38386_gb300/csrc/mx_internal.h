@@ -51,7 +51,9 @@ enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
 //   prefill: {ITEM_PREFILL, t | hq << 16, s | n_s << 16, partial slot base}
 //            piece s of n_s of query tile t (rows [128t, 128t+128)) of head hq;
 //            the tile's key tiles are split evenly between its n_s pieces.
-//   decode:  {ITEM_DECODE, decode index, kv head, split index}
+//   decode:  {ITEM_DECODE | kv head << 8 | split index << 16, decode index,
+//             page-table row, cached tokens}: the row and the length travel in
+//             the item so that the page-id loads need no other lookup first
 __host__ __device__ inline int4 prefill_item_code(int t, int hq, int s, int n_s, int part_base)
 {
     int4 r;
@@ -61,13 +63,13 @@ __host__ __device__ inline int4 prefill_item_code(int t, int hq, int s, int n_s,
     r.w = part_base;
     return r;
 }
-__host__ __device__ inline int4 decode_item_code(int i, int h, int s)
+__host__ __device__ inline int4 decode_item_code(int i, int h, int s, int seq, int ctx)
 {
     int4 r;
-    r.x = ITEM_DECODE;
+    r.x = ITEM_DECODE | (h << 8) | (s << 16);   // h < 256, s < 32768
     r.y = i;
-    r.z = h;
-    r.w = s;
+    r.z = seq;
+    r.w = ctx;
     return r;
 }
 

@@ -15,7 +15,7 @@
 //                           writes (O, lse) partials; the last-arriving piece
 //                           merges them.  Piece 0 of the head group's first
 //                           query head appends the tile's K/V.
-//   ITEM_DECODE  {i, h, s}: split s of decode i's keys for KV head h, all n_rep
+//   ITEM_DECODE  {h, s | i | seq | ctx}: split s of decode i's keys for KV head h, all n_rep
 //                           query heads of the group at once: a split-KV
 //                           flash-decode whose partial (O, lse) is merged by
 //                           the last-arriving split (no waiting).
@@ -98,11 +98,12 @@ __device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t
 }
 
 __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int di, int h,
-                            int s)
+                            int s, int seq, int n)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // split count and partial slots are needed only at the end: the load
+    // overlaps the page-id loads (the row and length came with the item)
     const DecodeInfo D = P.dec[di];
-    const int n = D.ctx;
     const int nrep = P.n_rep;
     const int k_lo = s * P.split_keys;
     const int k_hi = min(k_lo + P.split_keys, n + 1);
@@ -111,7 +112,7 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
     const int g = lane >> 2, tq = lane & 3;
 
     // The split holding the new key appends it (each slot written once).
-    if (s == D.n_splits - 1 && warp == 0) {
+    if (k_hi == n + 1 && warp == 0) {
         const int slot = P.slots[di];
         if (slot >= 0) {
             if (slot >= P.num_pages * kPage) {
@@ -152,7 +153,7 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
     if (lane < my_n) {
         const int lp = pg_lo + warp + kWarps * lane;
         if (lp * kPage < n) {  // pages holding cached keys only
-            int pid = __ldg(P.page_table + (size_t)D.seq * P.max_pages + lp);
+            int pid = __ldg(P.page_table + (size_t)seq * P.max_pages + lp);
             if (pid < 0 || pid >= P.num_pages) {
                 flag_error(P, ERR_PAGE);
                 pid = -1;
@@ -846,7 +847,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
                 merge_ns = ns;
             }
         } else {
-            decode_item(P, smem, misc, it.y, it.z, it.w);
+            decode_item(P, smem, misc, it.y, (it.x >> 8) & 0xFF, (int)((uint32_t)it.x >> 16), it.z, it.w);
         }
         fence_proxy_async_smem();  // generic smem accesses before later TMA writes
         tc_fence_before();
