@@ -328,6 +328,34 @@ def e2e_measure(w, steps, device):
             "seconds": dt, "copies": "pinned host <-> device, overlapped with compute on two copy streams"}
 
 
+def independent_layers_measure(w, steps, ws, device):
+    """The same steps with MX_OPT_PDL=2: layer l+1's CTAs start on the SMs
+    layer l frees.  The layers of this workload are independent problems, so
+    this is correct here, but a model whose layer l+1 reads layer l's output
+    cannot overlap them: the headline value keeps the dependent order."""
+    import torch
+
+    from paper_2609_38386_gb300 import MX_OPT_PDL
+    w.ctx.set_option(MX_OPT_PDL, 2)
+    try:
+        w.run_step()
+        torch.cuda.synchronize(device)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            w.run_step()
+        b.record()
+        torch.cuda.synchronize(device)
+        w.ctx.sync_status()
+        ms = max_over_ranks(a.elapsed_time(b), ws, device)
+    finally:
+        w.ctx.set_option(MX_OPT_PDL, 1)
+    return {"value": whole_job_value(w.tokens_per_step, steps, ws, ms), "unit": UNIT,
+            "ms_per_step": ms / steps,
+            "note": "MX_OPT_PDL=2: consecutive layers overlap (valid only for independent layers)"}
+
+
 # ------------------------------------------------------------- CPU oracle
 def oracle_sample(cfg, which="heavy"):
     """A bounded slice of the workload for the CPU oracle: one layer call of
@@ -667,6 +695,8 @@ def main():
             "plan_last": plan}
     if not args.no_e2e and not args.profile:
         line["e2e"] = e2e_measure(w, max(1, min(args.steps, 3)), device)
+    if not args.profile:
+        line["independent_layers"] = independent_layers_measure(w, args.steps, ws, device)
     if rank == 0 and ws == 1 and not args.no_cpu and not args.profile:
         line["cpu_baseline"] = cpu_baseline(cfg)
     if rank == 0:

@@ -171,10 +171,14 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
 #define MX_OPT_SPLIT_KEYS 1
 #define MX_OPT_GRID 2
 #define MX_OPT_PREFILL_PIECE_TILES 3
-/* MX_OPT_PDL: 1 (default) launches layers 2..L of mx_iteration with
- * programmatic dependent launch: a layer starts working on the SMs the
- * previous layer frees once that layer's work queue has drained (consecutive
- * launches use alternate workspace sets); 0 = ordinary stream order. */
+/* MX_OPT_PDL: how the layer launches of mx_iteration follow each other.
+ * 1 (default): programmatic dependent launch hides the launch latency, and
+ * layer l+1 starts working once layer l has finished: the order of a model
+ * whose layer l+1 attention reads what layer l produced.  2: the layers are
+ * independent problems; layer l+1's CTAs start on the SMs layer l frees,
+ * filling layer l's tail (needs a grid of every SM, else behaves as 1).
+ * 0: ordinary stream order.  Consecutive launches use three workspace sets
+ * in turn. */
 #define MX_OPT_PDL 4
 int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 

@@ -34,6 +34,11 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
 
 constexpr int kPlanSlots = 4;         // ring of work-list buffers
 constexpr int kPartSlots = 16384;     // decode split partials capacity
+// Workspace sets (counters, partials), used by consecutive launches in turn.
+// A launch lets its successor start as soon as its own CTAs are resident and
+// waits for its predecessor before it exits, so when launch n + 3 starts,
+// launch n has completed and its set is free again.
+constexpr int kWorkSets = 3;
 constexpr int kPrePartSlots = 1024;   // prefill piece partials capacity (64 KiB each)
 constexpr int kMinPieceTiles = 48;    // smallest prefill piece, in 128-key tiles
 constexpr int kMaxSplitKeys = kWarps * 32 * kPage;  // 4096: one page id per lane
@@ -57,7 +62,7 @@ struct mx_ctx {
         float *pre_o, *pre_lse;
         uint32_t *pre_cnt;
         uint32_t *work_cnt;
-    } set[2] = {};
+    } set[kWorkSets] = {};
     uint64_t launch_seq = 0;
     uint32_t *err = nullptr;
     uint8_t *plan_dev[kPlanSlots] = {};
@@ -74,7 +79,7 @@ struct mx_ctx {
     int split_keys_opt = 0;
     int grid_opt = 0;
     int piece_tiles_opt = 0;
-    bool pdl = true;  // programmatic dependent launch between layer kernels
+    int pdl = 1;  // MX_OPT_PDL: 0 stream order, 1 dependent layers, 2 independent layers
     // last plan
     int last_items = 0, last_split = 0, last_prefill_items = 0, last_piece_tiles = 0;
     std::string last_error;
@@ -352,7 +357,7 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->slots = d->slots;
     P->items = pl.items_dev;
     P->dec = pl.dec_dev;
-    const mx_ctx::Set &w = c->set[set & 1];
+    const mx_ctx::Set &w = c->set[set % kWorkSets];
     P->part_o = w.part_o;
     P->part_lse = w.part_lse;
     P->merge_cnt = w.merge_cnt;
@@ -504,11 +509,11 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     const size_t plan_stride = (c->plan_bytes + 255) & ~size_t(255);
     const size_t set_bytes = part_o_bytes + part_lse_bytes + ((merge_bytes + 255) & ~size_t(255)) +
                              pre_o_bytes + pre_lse_bytes + pre_cnt_bytes + 256 /*work counters*/;
-    const size_t total = 2 * set_bytes + 256 /*error word*/ + kPlanSlots * plan_stride;
+    const size_t total = kWorkSets * set_bytes + 256 /*error word*/ + kPlanSlots * plan_stride;
     if ((e = cudaMalloc(&c->ws, total)) != cudaSuccess)
         return bail(e, "cudaMalloc(workspace)");
     uint8_t *p = c->ws;
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < kWorkSets; ++k) {
         mx_ctx::Set &w = c->set[k];
         w.part_o = reinterpret_cast<float *>(p);
         p += part_o_bytes;
@@ -539,7 +544,7 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
         if ((e = cudaEventCreateWithFlags(&c->plan_ev[s], cudaEventDisableTiming)) != cudaSuccess)
             return bail(e, "cudaEventCreate");
     }
-    for (int k = 0; k < 2; ++k)
+    for (int k = 0; k < kWorkSets; ++k)
         if ((e = cudaMemset(c->set[k].merge_cnt, 0, merge_bytes)) != cudaSuccess ||
             (e = cudaMemset(c->set[k].pre_cnt, 0, pre_cnt_bytes)) != cudaSuccess ||
             (e = cudaMemset(c->set[k].work_cnt, 0, 256)) != cudaSuccess)
@@ -625,7 +630,7 @@ int mx_mixed_attention(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b,
     if ((rc = plan(c, d, st, &pl)))
         return rc;
     LayerParams P;
-    if ((rc = make_params(c, d, b, pl, &P, (int)(c->launch_seq & 1))))
+    if ((rc = make_params(c, d, b, pl, &P, (int)(c->launch_seq % kWorkSets))))
         return rc;
     // ordinary stream order: the caller's next or previous work may depend on it
     cudaError_t e = launch_mixed_layer(P, grid_for(c, pl), st, false);
@@ -657,7 +662,7 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     // all descriptors are encoded before the timed region starts
     std::vector<LayerParams> params(work ? n_layers : 0);
     for (int l = 0; work && l < n_layers; ++l)
-        if ((rc = make_params(c, d, layers + l, pl, &params[l], (int)((c->launch_seq + l) & 1))))
+        if ((rc = make_params(c, d, layers + l, pl, &params[l], (int)((c->launch_seq + l) % kWorkSets))))
             return rc;
     cudaError_t e;
     if (timed && (e = cudaEventRecord(c->ev_start, st)) != cudaSuccess)
@@ -666,7 +671,16 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     // l > 0 may start while layer l - 1 drains; the first layer keeps
     // ordinary stream order behind whatever the caller enqueued before.
     for (int l = 0; work && l < n_layers; ++l) {
-        e = launch_mixed_layer(params[l], grid_for(c, pl), st, c->pdl && l > 0);
+        // Mode 1: layer l+1 launches as layer l's CTAs run out of work and
+        // starts once layer l has completed (launch latency hidden, no
+        // overlap: the order a model whose layers depend on each other
+        // imposes).  Mode 2: layer l+1's CTAs start on the SMs layer l frees.
+        // That is safe only when a launch occupies every SM (one CTA per SM):
+        // then launch n + 3 cannot start before launch n has completed (see
+        // kWorkSets); smaller grids keep mode 1.
+        const int grid = grid_for(c, pl);
+        params[l].early_start = (c->pdl == 2 && grid == c->num_sms) ? 1 : 0;
+        e = launch_mixed_layer(params[l], grid, st, c->pdl != 0 && l > 0);
         if (e != cudaSuccess)
             return cuda_fail(c, e, "mixed_layer launch");
         ++c->launch_seq;
@@ -721,9 +735,9 @@ int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
         c->piece_tiles_opt = (int)value;
         return MX_OK;
     case MX_OPT_PDL:
-        if (value != 0 && value != 1)
-            return fail(c, MX_EINVAL, "MX_OPT_PDL is 0 or 1");
-        c->pdl = value != 0;
+        if (value < 0 || value > 2)
+            return fail(c, MX_EINVAL, "MX_OPT_PDL is 0, 1 or 2");
+        c->pdl = (int)value;
         return MX_OK;
     case MX_OPT_GRID:
         if (value < 0 || value > 65535)

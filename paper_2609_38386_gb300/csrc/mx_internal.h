@@ -117,6 +117,7 @@ struct LayerParams {
     int32_t num_pages, max_pages;
     int32_t split_keys;    // keys per decode split (multiple of 128)
     int32_t has_prefill;   // allocate TMEM only when prefill tiles exist
+    int32_t early_start;   // let the next launch start as soon as this one is resident
     float scale_log2;      // log2(e) / sqrt(head_dim)
     uint64_t timeout_ns;   // bound on every in-kernel wait
 };

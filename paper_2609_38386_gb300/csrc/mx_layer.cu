@@ -817,6 +817,13 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     // kernel), so work starts at once, beside the previous layer's tail.
     if (tid == 0)
         misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
+    // Independent layers (early_start): the next launch may start once every
+    // CTA of this one is resident; its CTAs take the SMs this grid frees, so
+    // the next layer's work fills this layer's tail.  Consecutive launches
+    // use different workspace sets (three in turn) and touch disjoint
+    // tensors.
+    if (P.early_start)
+        pdl_launch_dependents();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -858,12 +865,13 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         buf ^= 1;
     }
 
-    // Out of work: once the previous launch has completed (it has, long ago),
-    // let the next launch start on the SMs this grid is freeing.  The next
-    // launch reuses the workspace set of the previous one, which is why this
-    // CTA waits for it first.
+    // Out of work: wait until the previous launch has completed before
+    // exiting, so that when a later launch reuses that launch's workspace
+    // set, it is complete.  Dependent layers signal the next launch only now,
+    // so it runs after this one (its launch latency hidden).
     pdl_wait();
-    pdl_launch_dependents();
+    if (!P.early_start)
+        pdl_launch_dependents();
     if (misc->abort) {
         // give in-flight copies and MMAs time to land before TMEM is freed
         const uint64_t t0 = globaltimer_ns();

@@ -239,3 +239,31 @@ def test_prefill_pieces_deterministic_and_reusable():
     np.testing.assert_array_equal(r1["out"], r2["out"])
     _ok(case.check(r2))
     ctx.close()
+
+
+def test_iteration_independent_layers_mode_matches():
+    """MX_OPT_PDL=2 (layer l+1 starts on the SMs layer l frees) gives the
+    bit-identical outputs and KV pages of the default mode, on a plan large
+    enough for a grid of every SM, over several layers."""
+    from paper_2609_38386_gb300 import MX_OPT_PDL
+    rng = np.random.default_rng(12)
+    ctxs = [int(c) for c in rng.integers(1500, 4000, size=48)]
+    case = Case(16, ctxs, chunk_start=512, p_t=384, seed=21)
+    results = {}
+    for mode in (1, 2):
+        ctx = case.make_context()
+        ctx.set_option(MX_OPT_PDL, mode)
+        devs = [case.device_inputs() for _ in range(5)]
+        layers = [ctx.make_bufs(d["q"], d["k"], d["v"], d["k_pool"], d["v_pool"], d["out"]) for d in devs]
+        desc = case.desc(ctx, devs[0])
+        for _ in range(3):
+            ctx.iteration(desc, layers)
+        assert ctx.last_plan()["n_items"] >= torch.cuda.get_device_properties(0).multi_processor_count
+        results[mode] = [(d["out"].cpu().numpy(), d["k_pool"].cpu().numpy()) for d in devs]
+        ctx.close()
+    for (o1, k1), (o2, k2) in zip(results[1], results[2]):
+        np.testing.assert_array_equal(o1, o2)
+        np.testing.assert_array_equal(k1, k2)
+    ref = case.check({"out": results[2][0][0].view(np.uint16), "k_pool": results[2][0][1].view(np.uint16),
+                      "v_pool": devs[0]["v_pool"].cpu().numpy().view(np.uint16)})
+    _ok(ref)
