@@ -189,10 +189,20 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     int split = c->split_keys_opt;
     if (split <= 0) {
         // Each split pays a fixed start-up and merge cost, so splits are as long
-        // as load balance allows: about 1.5 per SM for a decode-only iteration,
-        // one per SM beside prefill tiles (which fill the rest of the launch).
-        const int64_t target_items = d->p_t > 0 ? (int64_t)c->num_sms : 3LL * c->num_sms / 2;
-        int64_t s = (total_keys + target_items - 1) / std::max<int64_t>(target_items, 1);
+        // as load balance allows: about 1.5 per SM for a decode-only iteration.
+        // Beside prefill tiles, which hold SMs from the start, the decode
+        // splits must fill around them: the fewer the query tiles, the finer
+        // (3 per SM beside 2 tiles, 2 beside 4, 1 from 6 on; a sweep of
+        // 1024-4096-key splits over the 0.6B sweep's chunk sizes put the
+        // optimum there).  With independent layers (MX_OPT_PDL = 2) the next
+        // layer fills the tail, so the splits stay long.
+        double per_sm = 1.5;
+        if (d->p_t > 0) {
+            const int n_qt = (d->p_t + kTileM - 1) / kTileM;
+            per_sm = c->pdl == 2 ? 1.0 : std::min(3.5, std::max(1.0, 3.5 - 0.5 * (n_qt - 1)));
+        }
+        const int64_t target_items = std::max<int64_t>(1, (int64_t)(per_sm * c->num_sms));
+        int64_t s = (total_keys + target_items - 1) / target_items;
         s = (s + 127) / 128 * 128;
         split = (int)std::min<int64_t>(std::max<int64_t>(s, 512), kMaxSplitKeys);
     }
@@ -278,13 +288,19 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         items[n++] = x.code;
     const int n_prefill = n;
 
+    // A decode with more keys than the split size is cut into equal
+    // page-aligned parts (no short remainder split: each split pays a fixed
+    // start-up and a merge).
     int part = 0;
-    struct DItem { int keys; int i, h, s; };
+    struct DItem { int keys; int i, h, s, len; };
     std::vector<DItem> ditems;
     ditems.reserve(64);
     for (int i = 0; i < nd; ++i) {
         const int keys = d->decode_ctx_lens[i] + 1;
         const int ns = (keys + split - 1) / split;
+        const int len = ((keys + ns - 1) / ns + kPage - 1) / kPage * kPage;
+        if (ns > kMaxDecodeSplits)
+            return fail(c, MX_ECAPACITY, "decode %d needs %d splits (limit %d)", i, ns, kMaxDecodeSplits);
         dec[i].seq = d->decode_seq_ids[i];
         dec[i].ctx = d->decode_ctx_lens[i];
         dec[i].n_splits = ns;
@@ -293,7 +309,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
             part += ns * hkv;
         for (int h = 0; h < hkv; ++h)
             for (int s = 0; s < ns; ++s)
-                ditems.push_back({std::min(split, keys - s * split), i, h, s});
+                ditems.push_back({std::min(len, keys - s * len), i, h, s, len});
     }
     if (n_prefill + (int)ditems.size() > c->max_items)
         return fail(c, MX_ECAPACITY, "work list of %zu items exceeds capacity %d",
@@ -301,7 +317,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     std::stable_sort(ditems.begin(), ditems.end(),
                      [](const DItem &a, const DItem &b) { return a.keys > b.keys; });
     for (const DItem &x : ditems)
-        items[n++] = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx);
+        items[n++] = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx, x.len);
 
     const size_t bytes = items_off + (size_t)n * sizeof(int4);
     // A kernel, not a copy engine, moves the plan: an H2D memcpy on the
@@ -464,7 +480,8 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     if (!out || !g)
         return MX_EINVAL;
     *out = nullptr;
-    if (g->head_dim != kHeadDim || g->page_size != kPage || g->num_kv_heads <= 0 || g->num_kv_heads > 255 ||
+    if (g->head_dim != kHeadDim || g->page_size != kPage || g->num_kv_heads <= 0 ||
+        g->num_kv_heads > kMaxDecodeKvHeads ||
         g->num_q_heads <= 0 || g->num_q_heads % g->num_kv_heads != 0 ||
         g->num_q_heads / g->num_kv_heads > kMaxRep || g->num_pages <= 0 || g->num_seqs <= 0 ||
         g->max_pages_per_seq <= 0 || g->max_tokens < 0 || g->max_decodes < 0 ||

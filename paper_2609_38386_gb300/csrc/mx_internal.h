@@ -51,9 +51,11 @@ enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
 //   prefill: {ITEM_PREFILL, t | hq << 16, s | n_s << 16, partial slot base}
 //            piece s of n_s of query tile t (rows [128t, 128t+128)) of head hq;
 //            the tile's key tiles are split evenly between its n_s pieces.
-//   decode:  {ITEM_DECODE | kv head << 8 | split index << 16, decode index,
-//             page-table row, cached tokens}: the row and the length travel in
-//             the item so that the page-id loads need no other lookup first
+//   decode:  {ITEM_DECODE | kv head << 4 | split index << 11 | split
+//             length / 16 << 23, decode index, page-table row, cached tokens}:
+//             split s of decode i covers keys [s * len, (s + 1) * len) of
+//             [0, ctx]; the row, length and split size travel in the item so
+//             that the page-id loads need no other lookup first
 __host__ __device__ inline int4 prefill_item_code(int t, int hq, int s, int n_s, int part_base)
 {
     int4 r;
@@ -63,10 +65,13 @@ __host__ __device__ inline int4 prefill_item_code(int t, int hq, int s, int n_s,
     r.w = part_base;
     return r;
 }
-__host__ __device__ inline int4 decode_item_code(int i, int h, int s, int seq, int ctx)
+constexpr int kMaxDecodeKvHeads = 127;   // item field widths: head 7 bits,
+constexpr int kMaxDecodeSplits = 4095;   // split index 12 bits, length/16 9 bits
+__host__ __device__ inline int4 decode_item_code(int i, int h, int s, int seq, int ctx, int split_len)
 {
     int4 r;
-    r.x = ITEM_DECODE | (h << 8) | (s << 16);   // h < 256, s < 32768
+    r.x = (int32_t)((uint32_t)ITEM_DECODE | ((uint32_t)h << 4) | ((uint32_t)s << 11) |
+                    ((uint32_t)(split_len / 16) << 23));
     r.y = i;
     r.z = seq;
     r.w = ctx;

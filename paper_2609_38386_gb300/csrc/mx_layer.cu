@@ -98,15 +98,15 @@ __device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t
 }
 
 __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int di, int h,
-                            int s, int seq, int n)
+                            int s, int seq, int n, int split_len)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     // split count and partial slots are needed only at the end: the load
     // overlaps the page-id loads (the row and length came with the item)
     const DecodeInfo D = P.dec[di];
     const int nrep = P.n_rep;
-    const int k_lo = s * P.split_keys;
-    const int k_hi = min(k_lo + P.split_keys, n + 1);
+    const int k_lo = s * split_len;
+    const int k_hi = min(k_lo + split_len, n + 1);
     const int pg_lo = k_lo / kPage;
     const int npg = (k_hi - k_lo + kPage - 1) / kPage;
     const int g = lane >> 2, tq = lane & 3;
@@ -854,7 +854,9 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
                 merge_ns = ns;
             }
         } else {
-            decode_item(P, smem, misc, it.y, (it.x >> 8) & 0xFF, (int)((uint32_t)it.x >> 16), it.z, it.w);
+            const uint32_t dx = (uint32_t)it.x;
+            decode_item(P, smem, misc, it.y, (int)((dx >> 4) & 0x7Fu), (int)((dx >> 11) & 0xFFFu), it.z, it.w,
+                        (int)(dx >> 23) * 16);
         }
         fence_proxy_async_smem();  // generic smem accesses before later TMA writes
         tc_fence_before();

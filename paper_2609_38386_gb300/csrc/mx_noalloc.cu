@@ -239,12 +239,12 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
         const int ns = dec[i].n_splits;
         for (int h = 0; h < hkv; ++h)
             for (int s = 0; s < ns - 1; ++s)
-                items[n++] = decode_item_code(i, h, s, dec[i].seq, dec[i].ctx);
+                items[n++] = decode_item_code(i, h, s, dec[i].seq, dec[i].ctx, split);
     }
     const int tail0 = n;
     for (int i = 0; i < nd; ++i)
         for (int h = 0; h < hkv; ++h)
-            items[n++] = decode_item_code(i, h, dec[i].n_splits - 1, dec[i].seq, dec[i].ctx);
+            items[n++] = decode_item_code(i, h, dec[i].n_splits - 1, dec[i].seq, dec[i].ctx, split);
     std::stable_sort(items + tail0, items + n, [&](const int4 &a, const int4 &c) {
         const int ka = dec[a.y].ctx + 1 - (dec[a.y].n_splits - 1) * split;   // .y: decode index
         const int kc = dec[c.y].ctx + 1 - (dec[c.y].n_splits - 1) * split;

@@ -245,7 +245,7 @@ def test_iteration_independent_layers_mode_matches():
     """MX_OPT_PDL=2 (layer l+1 starts on the SMs layer l frees) gives the
     bit-identical outputs and KV pages of the default mode, on a plan large
     enough for a grid of every SM, over several layers."""
-    from paper_2609_38386_gb300 import MX_OPT_PDL
+    from paper_2609_38386_gb300 import MX_OPT_PDL, MX_OPT_SPLIT_KEYS
     rng = np.random.default_rng(12)
     ctxs = [int(c) for c in rng.integers(1500, 4000, size=48)]
     case = Case(16, ctxs, chunk_start=512, p_t=384, seed=21)
@@ -253,6 +253,7 @@ def test_iteration_independent_layers_mode_matches():
     for mode in (1, 2):
         ctx = case.make_context()
         ctx.set_option(MX_OPT_PDL, mode)
+        ctx.set_option(MX_OPT_SPLIT_KEYS, 1024)   # the same plan in both modes
         devs = [case.device_inputs() for _ in range(5)]
         layers = [ctx.make_bufs(d["q"], d["k"], d["v"], d["k_pool"], d["v_pool"], d["out"]) for d in devs]
         desc = case.desc(ctx, devs[0])
