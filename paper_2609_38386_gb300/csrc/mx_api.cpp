@@ -69,8 +69,11 @@ struct mx_ctx {
     // pinned staging for the work list
     uint8_t *plan_host[kPlanSlots] = {};
     const void *plan_host_dev[kPlanSlots] = {};  // device view of plan_host (mapped pinned memory)
-    cudaEvent_t plan_ev[kPlanSlots] = {};
+    cudaEvent_t plan_ev[kPlanSlots] = {};    // upload of the slot done
     bool plan_ev_used[kPlanSlots] = {};
+    cudaEvent_t slot_done[kPlanSlots] = {};  // last kernel reading the slot done
+    bool slot_done_used[kPlanSlots] = {};
+    cudaStream_t up_stream = nullptr;        // plan uploads, off the caller's stream
     size_t plan_bytes = 0;
     int plan_next = 0;
     cudaEvent_t ev_start = nullptr, ev_end = nullptr;
@@ -320,16 +323,23 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         items[n++] = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx, x.len);
 
     const size_t bytes = items_off + (size_t)n * sizeof(int4);
-    // A kernel, not a copy engine, moves the plan: an H2D memcpy on the
-    // caller's stream would queue behind the caller's own large uploads (one
-    // copy engine per direction serves all streams in order).
-    cudaError_t e = launch_plan_upload(c->plan_host_dev[slot], c->plan_dev[slot], bytes, stream);
+    // A kernel, not a copy engine, moves the plan (an H2D memcpy would queue
+    // behind the caller's own large uploads: one copy engine per direction
+    // serves all streams in order), on the context's own stream so that it
+    // runs while the caller's stream is still busy with earlier work: it
+    // waits only for the last kernel that read this slot, and the caller's
+    // stream waits for it.
+    cudaError_t e = cudaSuccess;
+    if (c->slot_done_used[slot] && (e = cudaStreamWaitEvent(c->up_stream, c->slot_done[slot], 0)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaStreamWaitEvent(slot)");
+    e = launch_plan_upload(c->plan_host_dev[slot], c->plan_dev[slot], bytes, c->up_stream);
     if (e != cudaSuccess)
         return cuda_fail(c, e, "plan upload");
-    e = cudaEventRecord(c->plan_ev[slot], stream);
-    if (e != cudaSuccess)
+    if ((e = cudaEventRecord(c->plan_ev[slot], c->up_stream)) != cudaSuccess)
         return cuda_fail(c, e, "cudaEventRecord(plan)");
     c->plan_ev_used[slot] = true;
+    if ((e = cudaStreamWaitEvent(stream, c->plan_ev[slot], 0)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaStreamWaitEvent(plan)");
 
     out->n_items = n;
     out->n_prefill = n_prefill;
@@ -435,6 +445,17 @@ int grid_for(const mx_ctx *c, const Plan &pl)
 {
     int grid = c->grid_opt > 0 ? c->grid_opt : c->num_sms;
     return std::max(1, std::min(grid, pl.n_items));
+}
+
+// The plan slot may be rewritten once the kernels enqueued on `st` so far
+// (the last ones reading it) have finished.
+int release_slot(mx_ctx *c, const Plan &pl, cudaStream_t st)
+{
+    cudaError_t e = cudaEventRecord(c->slot_done[pl.slot], st);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventRecord(slot)");
+    c->slot_done_used[pl.slot] = true;
+    return MX_OK;
 }
 
 int read_error_word(mx_ctx *c)
@@ -558,7 +579,8 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
         if ((e = cudaHostGetDevicePointer(&dv, c->plan_host[s], 0)) != cudaSuccess)
             return bail(e, "cudaHostGetDevicePointer(plan)");
         c->plan_host_dev[s] = dv;
-        if ((e = cudaEventCreateWithFlags(&c->plan_ev[s], cudaEventDisableTiming)) != cudaSuccess)
+        if ((e = cudaEventCreateWithFlags(&c->plan_ev[s], cudaEventDisableTiming)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&c->slot_done[s], cudaEventDisableTiming)) != cudaSuccess)
             return bail(e, "cudaEventCreate");
     }
     for (int k = 0; k < kWorkSets; ++k)
@@ -571,6 +593,8 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     if ((e = cudaEventCreate(&c->ev_start)) != cudaSuccess ||
         (e = cudaEventCreate(&c->ev_end)) != cudaSuccess)
         return bail(e, "cudaEventCreate");
+    if ((e = cudaStreamCreateWithFlags(&c->up_stream, cudaStreamNonBlocking)) != cudaSuccess)
+        return bail(e, "cudaStreamCreate");
 
     void *fn = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -597,7 +621,11 @@ int mx_destroy(mx_ctx *c)
             cudaFreeHost(c->plan_host[s]);
         if (c->plan_ev[s])
             cudaEventDestroy(c->plan_ev[s]);
+        if (c->slot_done[s])
+            cudaEventDestroy(c->slot_done[s]);
     }
+    if (c->up_stream)
+        cudaStreamDestroy(c->up_stream);
     if (c->ev_start)
         cudaEventDestroy(c->ev_start);
     if (c->ev_end)
@@ -654,7 +682,7 @@ int mx_mixed_attention(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b,
     if (e != cudaSuccess)
         return cuda_fail(c, e, "mixed_layer launch");
     ++c->launch_seq;
-    return MX_OK;
+    return release_slot(c, pl, st);
 }
 
 int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_layer_bufs *layers,
@@ -702,6 +730,8 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
             return cuda_fail(c, e, "mixed_layer launch");
         ++c->launch_seq;
     }
+    if (work && (rc = release_slot(c, pl, st)))
+        return rc;
     if (!timed)
         return MX_OK;
     if ((e = cudaEventRecord(c->ev_end, st)) != cudaSuccess)
