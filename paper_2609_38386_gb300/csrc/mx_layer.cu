@@ -33,8 +33,9 @@ struct Misc {
     uint64_t bar_q;
     uint64_t bar_kfull[kKStages];
     uint64_t bar_kempty[kKStages];
-    uint64_t bar_vfull[kVStages];
     uint64_t bar_sfull[2];
+    // P_b written (128 softmax arrivals) and V tile b landed (the V
+    // producer's arrive + transaction bytes): the one wait before P_b V_b
     uint64_t bar_pfull[2];
     uint64_t bar_odone[2];  // P.V of P buffer b done; frees P buffer b and V stage b
     uint32_t tmem_base;
@@ -43,7 +44,7 @@ struct Misc {
     int32_t last;
 };
 static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
-static_assert(kVStages == 2, "V stage c % 2 is released by the odone barrier of P buffer c & 1");
+static_assert(kVStages == 2, "V stage c % 2 shares the pfull and odone barriers of P buffer c & 1");
 
 // Instruction descriptors: S = Q K^T (both K-major) and O = P V (V MN-major).
 constexpr uint32_t kIdescS = idesc_bf16_f32(128, 128, false, false);
@@ -395,7 +396,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         const uint32_t ring = isK ? sK : sV;
         const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
         const void *tm_in = isK ? (const void *)&P.tm_k : (const void *)&P.tm_v;
-        uint64_t *full = isK ? misc->bar_kfull : misc->bar_vfull;
+        uint64_t *full = isK ? misc->bar_kfull : misc->bar_pfull;
         // V stage c % 2 is free once P_{c-2} V_{c-2} has completed, which is
         // exactly the odone barrier of P buffer c & 1 (one commit fewer per tile).
         uint64_t *empty = isK ? misc->bar_kempty : misc->bar_odone;
@@ -489,8 +490,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                     const int j = i - 1;
                     const uint32_t c = tile0 + j;
                     const int st = c % kVStages;
-                    if (!mbar_wait(smem_u32(&misc->bar_pfull[c & 1]), (c >> 1) & 1, abort, tmo) ||
-                        !mbar_wait(smem_u32(&misc->bar_vfull[st]), (c / kVStages) & 1, abort, tmo)) {
+                    if (!mbar_wait(smem_u32(&misc->bar_pfull[c & 1]), (c >> 1) & 1, abort, tmo)) {
                         ok = false;
                         break;
                     }
@@ -790,12 +790,9 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
             mbar_init(smem_u32(&misc->bar_kempty[b]), 1);
         }
-        for (int b = 0; b < kVStages; ++b) {
-            mbar_init(smem_u32(&misc->bar_vfull[b]), 1);
-        }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&misc->bar_sfull[b]), 1);
-            mbar_init(smem_u32(&misc->bar_pfull[b]), 128);
+            mbar_init(smem_u32(&misc->bar_pfull[b]), 128 + 1);
             mbar_init(smem_u32(&misc->bar_odone[b]), 1);
         }
         misc->abort = 0;
