@@ -245,7 +245,9 @@ def e2e_measure(w, steps, device):
     iterations the way a serving loop would run them: the inputs of iteration
     i+1 and i+2 upload on one stream and the outputs of iteration i-1
     download on another while iteration i computes (three device buffer
-    sets, so that a large iteration's upload has two iterations of slack)."""
+    sets, so that a large iteration's upload has two iterations of slack);
+    the pipeline runs across the timed steps and the region ends when the
+    last step's outputs are on the host."""
     import torch
     g, L = w.geom, w.L
     per_tok_in = (g.hq + 2 * g.hkv) * g.head_dim
@@ -291,41 +293,45 @@ def e2e_measure(w, steps, device):
     down = torch.cuda.Stream(device)
     n_it = len(w.its)
 
-    def one_step():
-        ev_in = [torch.cuda.Event() for _ in range(n_it)]
-        ev_comp = [torch.cuda.Event() for _ in range(n_it)]
-        ev_out = [torch.cuda.Event() for _ in range(n_it)]
-        for i in range(n_it):
-            b = i % nbuf
+    def run(n_steps):
+        # one continuous pipeline over the steps' iterations: iteration j uses
+        # buffer set j % nbuf, uploads as soon as iteration j - nbuf has
+        # consumed that set, and downloads as soon as it has computed
+        total = n_steps * n_it
+        ev_in = [torch.cuda.Event() for _ in range(total)]
+        ev_comp = [torch.cuda.Event() for _ in range(total)]
+        ev_out = [torch.cuda.Event() for _ in range(total)]
+        for j in range(total):
+            i, b = j % n_it, j % nbuf
             with torch.cuda.stream(up):
-                if i >= nbuf:
-                    up.wait_event(ev_comp[i - nbuf])   # inputs of i-nbuf consumed
+                if j >= nbuf:
+                    up.wait_event(ev_comp[j - nbuf])   # inputs of j-nbuf consumed
                 d_in[b][:in_elems[i]].copy_(h_in[:in_elems[i]], non_blocking=True)
-                ev_in[i].record(up)
-            comp.wait_event(ev_in[i])
-            if i >= nbuf:
-                comp.wait_event(ev_out[i - nbuf])      # outputs of i-nbuf downloaded
+                ev_in[j].record(up)
+            comp.wait_event(ev_in[j])
+            if j >= nbuf:
+                comp.wait_event(ev_out[j - nbuf])      # outputs of j-nbuf downloaded
             w.ctx.iteration(w.descs[i], layer_arrays[i][b], stream=comp, wait=False)
-            ev_comp[i].record(comp)
+            ev_comp[j].record(comp)
             with torch.cuda.stream(down):
-                down.wait_event(ev_comp[i])
+                down.wait_event(ev_comp[j])
                 h_out[:out_elems[i]].copy_(d_out[b][:out_elems[i]], non_blocking=True)
-                ev_out[i].record(down)
+                ev_out[j].record(down)
         for s_ in (up, comp, down):
             s_.synchronize()
 
-    one_step()  # warm-up
+    run(1)  # warm-up
     w.ctx.sync_status()
     torch.cuda.synchronize(device)
     t0 = time.perf_counter()
-    for _ in range(steps):
-        one_step()
+    run(steps)
     torch.cuda.synchronize(device)
     dt = time.perf_counter() - t0
     w.ctx.sync_status()
     return {"value": w.tokens_per_step * steps / dt, "unit": UNIT,
             "h2d_bytes_per_step": int(sum(in_elems) * 2), "d2h_bytes_per_step": int(sum(out_elems) * 2),
-            "seconds": dt, "copies": "pinned host <-> device, overlapped with compute on two copy streams"}
+            "seconds": dt, "copies": "pinned host <-> device on two copy streams, pipelined with "
+            "compute across the timed steps (every step's inputs and outputs inside the region)"}
 
 
 def independent_layers_measure(w, steps, ws, device):

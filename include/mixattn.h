@@ -72,7 +72,7 @@ typedef struct mx_ctx mx_ctx;
  * page-table shape. */
 typedef struct {
     int32_t num_q_heads;       /* Hq: 16, 32 or 64 in the Qwen3 geometries */
-    int32_t num_kv_heads;      /* Hkv: 8 (1..255; Hq / Hkv a power of two
+    int32_t num_kv_heads;      /* Hkv: 8 (1..127; Hq / Hkv a power of two
                                   of at most 8)                           */
     int32_t head_dim;          /* must be 128                             */
     int32_t page_size;         /* must be 16                              */

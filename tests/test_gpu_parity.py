@@ -268,3 +268,13 @@ def test_iteration_independent_layers_mode_matches():
     ref = case.check({"out": results[2][0][0].view(np.uint16), "k_pool": results[2][0][1].view(np.uint16),
                       "v_pool": devs[0]["v_pool"].cpu().numpy().view(np.uint16)})
     _ok(ref)
+
+
+@pytest.mark.parametrize("split", [0, 512])
+def test_decode_long_contexts_equal_parts(split):
+    """Decodes long enough to be cut into many equal page-aligned parts
+    (65 parts at a 512-key split), merged by log-sum-exp, beside short ones."""
+    from paper_2609_38386_gb300 import MX_OPT_SPLIT_KEYS
+    case = Case(32, [33000, 17, 4100, 513], seed=40 + split)
+    res = case.run_gpu(options={MX_OPT_SPLIT_KEYS: split} if split else None)
+    _ok(case.check(res))
