@@ -40,10 +40,12 @@ constexpr int kDecStages = 3;
 static_assert(kWarps * kDecStages * kDecStageBytes <= kSmemData, "decode ring too large");
 
 // TMEM columns: S buffers [0,128) and [128,256) (fp32), O [256,384) (fp32),
-// P buffers [384,448) and [448,512) (bf16 pairs, the A operand of P.V).
+// Q [384,448) (bf16 pairs, the A operand of Q.K^T).  P_b (bf16 pairs, the A
+// operand of P.V) overwrites the first 64 columns of S_b once they are read,
+// so that both MMAs read only K or V from shared memory.
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemO = 256;
-constexpr uint32_t kTmemP = 384;
+constexpr uint32_t kTmemQ = 384;
 
 enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
 

@@ -13,8 +13,9 @@
 //                           tiles, on tcgen05 tensor cores (S and O
 //                           accumulators in TMEM).  A tile with several pieces
 //                           writes (O, lse) partials; the last-arriving piece
-//                           merges them.  Piece 0 of the head group's first
-//                           query head appends the tile's K/V.
+//                           merges them.  Piece 0 of each of the n_rep
+//                           query heads of a KV head appends 128 / n_rep of
+//                           the tile's tokens to the KV cache.
 //   ITEM_DECODE  {h, s | i | seq | ctx}: split s of decode i's keys for KV head h, all n_rep
 //                           query heads of the group at once: a split-KV
 //                           flash-decode whose partial (O, lse) is merged by
@@ -361,6 +362,47 @@ __device__ __forceinline__ void clear_uncached_rows(uint32_t dv, int r0)
     fence_proxy_async_smem();
 }
 
+// Row max of the raw scores of one S row held in registers (the scale is
+// positive), 8 independent three-input chains.
+__device__ __forceinline__ float row_max(const uint32_t (&sv)[128])
+{
+    float mx8[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+        mx8[u] = neg_inf();
+#pragma unroll
+    for (int cc = 0; cc < 64; ++cc) {
+        mx8[cc & 7] = max3(mx8[cc & 7], __uint_as_float(sv[2 * cc]), __uint_as_float(sv[2 * cc + 1]));
+    }
+    return fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                 fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+}
+
+// p = 2^(s*scale - m) of one S row as bf16 pairs into TMEM at taddr (64
+// columns), and the row sum of p in 4 packed pair chains.
+__device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float sl, float nm, uint32_t taddr)
+{
+    float rs8[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+        rs8[u] = 0.f;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int cc = 0; cc < 32; ++cc) {
+            const int k0 = 64 * half + 2 * cc;
+            float x0, x1;
+            ffma2(x0, x1, __uint_as_float(sv[k0]), __uint_as_float(sv[k0 + 1]), sl, sl, nm, nm);
+            const float e0 = ex2(x0), e1 = ex2(x1);
+            fadd2(rs8[2 * (cc & 3)], rs8[2 * (cc & 3) + 1], e0, e1);
+            pk[cc] = pack_bf16(e0, e1);
+        }
+        tmem_st32(taddr + 32 * half, pk);
+    }
+    return ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
+}
+
 // ---------------------------------------------------------------------------
 // Prefill tile: rows [128t, 128t + 128) of the chunk, query head hq.
 // Key tiles: nA paged tiles covering [0, chunk_start), then t + 1 tiles of
@@ -376,7 +418,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
     const int nA = (cs + kTileN - 1) / kTileN;
     const int nT = kt1 - kt0;  // key tiles of this piece: global tiles kt0 + i
     const uint32_t sbase = smem_u32(smem);
-    const uint32_t sQ = sbase + kSmemQ, sK = sbase + kSmemK, sV = sbase + kSmemV;
+    const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;
     const uint32_t bar_q = smem_u32(&misc->bar_q);
     volatile int *abort = &misc->abort;
     const uint64_t tmo = P.timeout_ns;
@@ -386,12 +428,6 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         // warp 0 loads Q and the K tiles, warp 3 the V tiles; each waits only
         // on its own ring's "empty" barriers.
         const bool isK = warp == 0;
-        if (isK && lane == 0) {
-            fence_proxy_async_smem();
-            mbar_expect_tx(bar_q, kTileBytes);
-            tma_load_3d(sQ, &P.tm_q, bar_q, 0, hq, nd + kTileM * t);
-            tma_load_3d(sQ + kHalfTile, &P.tm_q, bar_q, 64, hq, nd + kTileM * t);
-        }
         const int nst = isK ? kKStages : kVStages;
         const uint32_t ring = isK ? sK : sV;
         const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
@@ -401,29 +437,38 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         // exactly the odone barrier of P buffer c & 1 (one commit fewer per tile).
         uint64_t *empty = isK ? misc->bar_kempty : misc->bar_odone;
         const int oob_row = P.num_pages * P.hkv * kPage;
+        // Page ids of cached tiles, four tiles (32 pages, one per lane) per
+        // load, fetched one batch ahead: a page-table read under load takes
+        // about as long as a whole tile, so it must not sit in the issue loop.
+        const int32_t *prow = P.page_table + (size_t)P.prefill_seq * P.max_pages;
+        auto fetch_pids = [&](int i0) {
+            const int lp = (kt0 + i0 + (lane >> 3)) * 8 + (lane & 7);
+            int pid = -1;
+            if (i0 + (lane >> 3) < nT && lp * kPage < cs) {
+                pid = __ldg(prow + lp);
+                if (pid < 0 || pid >= P.num_pages) {
+                    if (isK)
+                        flag_error(P, ERR_PAGE);
+                    pid = -1;
+                }
+            }
+            return pid;
+        };
+        int pid_cur = fetch_pids(0), pid_next = fetch_pids(4);
         for (int i = 0; i < nT; ++i) {
             const uint32_t c = tile0 + i;
             const int st = c % nst;
             const uint32_t ph = (c / nst) & 1;
             const int gi = kt0 + i;
             const bool paged = gi < nA;
-            int pid_l = -1;
-            if (paged && lane < 8) {
-                const int lp = gi * 8 + lane;
-                if (lp * kPage < cs) {
-                    int pid = __ldg(P.page_table + (size_t)P.prefill_seq * P.max_pages + lp);
-                    if (pid < 0 || pid >= P.num_pages) {
-                        if (isK)
-                            flag_error(P, ERR_PAGE);
-                        pid = -1;
-                    }
-                    pid_l = pid;
-                }
+            if (i > 0 && (i & 3) == 0) {
+                pid_cur = pid_next;
+                pid_next = fetch_pids(i + 4);
             }
             int pids[8];
 #pragma unroll
             for (int pg = 0; pg < 8; ++pg)
-                pids[pg] = __shfl_sync(0xffffffffu, pid_l, pg);
+                pids[pg] = __shfl_sync(0xffffffffu, pid_cur, (i & 3) * 8 + pg);
             int ok = 1;
             if (lane == 0) {
                 if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1, abort, tmo)) {
@@ -474,14 +519,14 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                         break;
                     }
                     tc_fence_after();
-                    const uint64_t qdesc = smem_desc(sQ, 16, 1024, kSwz128);
                     const uint64_t kdesc = smem_desc(sK + st * kTileBytes, 16, 1024, kSwz128);
                     const uint32_t d = tmem + (c & 1) * 128;
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
-                        // 16 keys of K-major SW128: +32 B inside a 64-column half
+                        // 16 dims: 8 columns of Q in TMEM; +32 B inside a
+                        // 64-column half of the K-major SW128 K tile
                         const uint64_t off = (uint64_t)(((kk >> 2) * kHalfTile + (kk & 3) * 32) >> 4);
-                        tc_mma_ss(d, qdesc + off, kdesc + off, kIdescS, kk > 0 ? 1u : 0u);
+                        tc_mma_ts(d, tmem + kTmemQ + kk * 8, kdesc + off, kIdescS, kk > 0 ? 1u : 0u);
                     }
                     tc_commit(smem_u32(&misc->bar_sfull[c & 1]));
                     tc_commit(smem_u32(&misc->bar_kempty[st]));
@@ -499,7 +544,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                         clear_uncached_rows(dv, cs - (kt0 + j) * kTileN);
                     tc_fence_after();
                     const uint64_t vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
-                    const uint32_t pa = tmem + kTmemP + (c & 1) * 64;  // P_c: 8 columns per 16 keys
+                    const uint32_t pa = tmem + (c & 1) * 128;  // P_c over S_c: 8 columns per 16 keys
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk)  // 16 keys of MN-major V: +2 KiB
                         tc_mma_ts(tmem + kTmemO, pa + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4), kIdescO,
@@ -511,56 +556,70 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 set_abort(P, misc);
         }
         __syncwarp();
-    } else if (warp == 2) {
-        // ------------------------------------------------ chunk KV append
-        // The n_rep query heads of a KV head share its 128 tokens: head r of
-        // the group appends tokens [r*128/n_rep, (r+1)*128/n_rep) of the tile.
-        // 16 tokens per round so that 16 loads per lane are in flight.
-        if (kt0 == 0) {
-            const int per = kTileM / P.n_rep;
-            const int j0 = kTileM * t + (hq % P.n_rep) * per;
-            const int ntok = min(per, p - j0);
-            constexpr int U = 16;
-            const int c16 = lane & 15;
-            const bool isv = lane >= 16;
-            const uint16_t *src_base = isv ? P.v : P.k;
-            uint16_t *dst_base = isv ? P.v_pool : P.k_pool;
-            for (int tb = 0; tb < ntok; tb += U) {
-                int my_slot = -1;
-                if (lane < U && tb + lane < ntok)
-                    my_slot = __ldg(P.slots + nd + j0 + tb + lane);
-                uint4 val[U];
-                int sl[U];
-#pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    sl[u] = __shfl_sync(0xffffffffu, my_slot, u);
-                    if (tb + u < ntok && sl[u] >= 0 && sl[u] < P.num_pages * kPage) {
-                        const size_t src = ((size_t)(nd + j0 + tb + u) * P.hkv + kvh) * kHeadDim;
-                        val[u] = __ldg(reinterpret_cast<const uint4 *>(src_base + src) + c16);
-                    }
-                }
-#pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    if (tb + u >= ntok || sl[u] < 0)
-                        continue;
-                    if (sl[u] >= P.num_pages * kPage) {
-                        if (lane == 0)
-                            flag_error(P, ERR_SLOT);
-                        continue;
-                    }
-                    const size_t dst =
-                        (((size_t)(sl[u] / kPage) * P.hkv + kvh) * kPage + sl[u] % kPage) * kHeadDim;
-                    reinterpret_cast<uint4 *>(dst_base + dst)[c16] = val[u];
-                }
-            }
-        }
-    } else {
+    } else if (warp >= 4) {
         // ------------------------------------------------ softmax / epilogue
         const int q4 = warp - 4;
         const int r = q4 * 32 + lane;          // tile row = TMEM lane
         const int j = kTileM * t + r;          // chunk row offset
         const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
         const float sl = P.scale_log2;
+        {
+            // Q row j of head hq into TMEM lane r (zeros past the chunk's end).
+            // Piece 0 also appends this head's share of the tile's K/V: the
+            // n_rep query heads of a KV head split its 128 tokens (head r of
+            // the group takes tokens [r*128/n_rep, (r+1)*128/n_rep)), and the
+            // 32 16-byte pieces of a token's K and V rows are split between
+            // n_rep threads.  The append's loads go out with Q's, so that one
+            // memory latency covers both.
+            uint32_t qv[64];
+            const uint4 *qrow = reinterpret_cast<const uint4 *>(P.q + ((size_t)(nd + j) * P.hq + hq) * kHeadDim);
+#pragma unroll
+            for (int x = 0; x < 16; ++x) {
+                const uint4 v4 = j < p ? __ldg(qrow + x) : make_uint4(0u, 0u, 0u, 0u);
+                qv[4 * x] = v4.x;
+                qv[4 * x + 1] = v4.y;
+                qv[4 * x + 2] = v4.z;
+                qv[4 * x + 3] = v4.w;
+            }
+            const int per = kTileM / P.n_rep, npc = 32 / P.n_rep;
+            const int u = r / P.n_rep, sub = r % P.n_rep;
+            const int ja = kTileM * t + (hq % P.n_rep) * per + u;   // chunk row of this thread's token
+            const bool app = kt0 == 0 && ja < p;
+            const size_t arow = ((size_t)(nd + ja) * P.hkv + kvh) * kHeadDim;
+            int slot = -1;
+            if (app)
+                slot = __ldg(P.slots + nd + ja);
+            for (int b = 0; b < npc; b += 16) {
+                uint4 av[16];
+#pragma unroll
+                for (int x = 0; x < 16; ++x) {
+                    const int pc = sub * npc + b + x;   // piece: K row 0..15, V row 16..31
+                    if (app && x < npc - b)
+                        av[x] = __ldg(reinterpret_cast<const uint4 *>((pc < 16 ? P.k : P.v) + arow) + (pc & 15));
+                }
+                if (b == 0) {
+                    tmem_st32(tl + kTmemQ, *reinterpret_cast<uint32_t(*)[32]>(&qv[0]));
+                    tmem_st32(tl + kTmemQ + 32, *reinterpret_cast<uint32_t(*)[32]>(&qv[32]));
+                    tmem_wait_st();
+                    tc_fence_before();
+                    mbar_arrive(bar_q);
+                }
+                if (app && slot >= 0) {
+                    if (slot >= P.num_pages * kPage) {
+                        if (sub == 0 && b == 0)
+                            flag_error(P, ERR_SLOT);
+                    } else {
+                        const size_t dst = (((size_t)(slot / kPage) * P.hkv + kvh) * kPage + slot % kPage) * kHeadDim;
+#pragma unroll
+                        for (int x = 0; x < 16; ++x) {
+                            const int pc = sub * npc + b + x;
+                            if (x < npc - b)
+                                reinterpret_cast<uint4 *>((pc < 16 ? P.k_pool : P.v_pool) + dst)[pc & 15] = av[x];
+                        }
+                    }
+                }
+            }
+        }
         float m_run = neg_inf(), l_run = 0.f;
         bool ok = true;
         for (int i = 0; i < nT; ++i) {
@@ -574,40 +633,30 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             const int gi = kt0 + i;
             const int nvalid = gi < nA ? min(kTileN, cs - gi * kTileN)
                                        : min(kTileN, j - kTileN * (gi - nA) + 1);
-            // Pass 1: row max of the raw scores (the scale is positive) over
-            // the two 64-column halves of S, 8 independent three-input chains.  S is read
-            // from TMEM twice (here and in pass 2) to keep only 64 scores live.
-            float mx8[8];
+            // Row r of S_c: all 128 raw scores read from TMEM once (a second
+            // read would compete with the tensor core's own TMEM traffic).
+            uint32_t sv[128];
 #pragma unroll
-            for (int u = 0; u < 8; ++u)
-                mx8[u] = neg_inf();
+            for (int q = 0; q < 4; ++q)
+                tmem_ld32(tl + sb * 128 + 32 * q, *reinterpret_cast<uint32_t(*)[32]>(&sv[32 * q]));
+            tmem_wait_ld();
+            if (nvalid < kTileN) {  // boundary tiles only: masked keys -> -inf
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                uint32_t sv[64];
-                tmem_ld32(tl + sb * 128 + 64 * half, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
-                tmem_ld32(tl + sb * 128 + 64 * half + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
-                tmem_wait_ld();
-                if (nvalid < kTileN) {  // boundary tiles only: masked keys -> -inf
-#pragma unroll
-                    for (int cc = 0; cc < 64; ++cc)
-                        if (64 * half + cc >= nvalid)
-                            sv[cc] = 0xFF800000u;
-                }
-#pragma unroll
-                for (int cc = 0; cc < 32; ++cc)
-                    mx8[cc & 7] = max3(mx8[cc & 7], __uint_as_float(sv[2 * cc]), __uint_as_float(sv[2 * cc + 1]));
+                for (int cc = 0; cc < 128; ++cc)
+                    if (cc >= nvalid)
+                        sv[cc] = 0xFF800000u;
             }
-            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+            const float mx = row_max(sv);
             const float m_new = fmaxf(m_run, mx * sl);   // log2 domain
             const bool rescale = m_new > m_run + 8.0f;
             const float m_use = rescale ? m_new : m_run;
             const float nm = -m_use;
-            // P buffer (c & 1) was last read by tile c - 2's PV.
-            if (i >= 2 && !mbar_wait(smem_u32(&misc->bar_odone[c & 1]), ((c - 2) >> 1) & 1, abort, tmo)) {
-                ok = false;
-                break;
-            }
+            // P_c (the A operand of P.V) goes over the first 64 columns of
+            // S_c, whose buffer P_{c-2} held: S_c was issued after
+            // P_{c-2} V_{c-2}, so its completion covers that read too.
+            const float rs = row_exp_store(sv, sl, nm, tl + sb * 128);
+            // The O correction comes after P, when the scores are no longer
+            // live, and before P_c is released to the MMA issuer.
             if (rescale && i > 0) {
                 // O must be stable: tile c - 1's PV has completed.
                 if (!mbar_wait(smem_u32(&misc->bar_odone[(c - 1) & 1]), ((c - 1) >> 1) & 1, abort, tmo)) {
@@ -629,36 +678,6 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                 tmem_wait_st();
                 l_run *= alpha;
             }
-            // Pass 2: p = 2^(s*scale - m) as bf16 pairs into TMEM lane r (the A
-            // operand of P.V), and the row sum in 4 packed pair chains.
-            float rs8[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u)
-                rs8[u] = 0.f;
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                uint32_t sv[64];
-                tmem_ld32(tl + sb * 128 + 64 * half, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
-                tmem_ld32(tl + sb * 128 + 64 * half + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
-                tmem_wait_ld();
-                if (nvalid < kTileN) {
-#pragma unroll
-                    for (int cc = 0; cc < 64; ++cc)
-                        if (64 * half + cc >= nvalid)
-                            sv[cc] = 0xFF800000u;
-                }
-                uint32_t pk[32];
-#pragma unroll
-                for (int cc = 0; cc < 32; ++cc) {
-                    float x0, x1;
-                    ffma2(x0, x1, __uint_as_float(sv[2 * cc]), __uint_as_float(sv[2 * cc + 1]), sl, sl, nm, nm);
-                    const float e0 = ex2(x0), e1 = ex2(x1);
-                    fadd2(rs8[2 * (cc & 3)], rs8[2 * (cc & 3) + 1], e0, e1);
-                    pk[cc] = pack_bf16(e0, e1);
-                }
-                tmem_st32(tl + kTmemP + (c & 1) * 64 + 32 * half, pk);
-            }
-            const float rs = ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
             l_run += rs;
             m_run = m_use;
             tmem_wait_st();
@@ -785,7 +804,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     const int tid = threadIdx.x, warp = tid >> 5;
 
     if (tid == 0) {
-        mbar_init(smem_u32(&misc->bar_q), 1);
+        mbar_init(smem_u32(&misc->bar_q), 128);
         for (int b = 0; b < kKStages; ++b) {
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
             mbar_init(smem_u32(&misc->bar_kempty[b]), 1);
@@ -798,7 +817,6 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         misc->abort = 0;
         fence_mbar_init();
         if (P.has_prefill) {
-            tma_prefetch_desc(&P.tm_q);
             tma_prefetch_desc(&P.tm_k);
             tma_prefetch_desc(&P.tm_v);
             tma_prefetch_desc(&P.tm_kpool);
