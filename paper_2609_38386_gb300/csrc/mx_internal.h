@@ -21,14 +21,15 @@ constexpr int kTileN = 128;
 // Shared-memory plan (bytes, offsets from a 1024-aligned base).
 constexpr int kHalfTile = kTileM * 64 * 2;             // 128 rows x 64 bf16 = 16 KiB
 constexpr int kTileBytes = 2 * kHalfTile;              // 32 KiB
-// K tiles are released as soon as S = Q K^T has completed and V tiles after
-// P V, so K gets the deeper ring: a K load is issued ~4 tiles before use.
-constexpr int kKStages = 4;
+// K stage c % 3 is released by the completion of S_c = Q K_c^T (the same
+// barrier that hands S_c to the softmax) and V stage c % 2 by that of P_c V_c;
+// the loads run two to three tiles ahead of their use.
+constexpr int kKStages = 3;
 constexpr int kVStages = 2;
 constexpr int kSmemQ = 0;
 constexpr int kSmemK = kSmemQ + kTileBytes;
 constexpr int kSmemV = kSmemK + kKStages * kTileBytes;
-constexpr int kSmemData = kSmemV + kVStages * kTileBytes;   // 224 KiB
+constexpr int kSmemData = kSmemV + kVStages * kTileBytes;   // 192 KiB
 constexpr int kSmemMisc = kSmemData;                   // barriers etc.
 constexpr int kSmemMiscBytes = 1024;
 constexpr int kSmemTotal = kSmemData + kSmemMiscBytes + 1024;  // + alignment slack
@@ -39,13 +40,13 @@ constexpr int kDecStageBytes = 2 * kPageBytes;         // 8 KiB
 constexpr int kDecStages = 3;
 static_assert(kWarps * kDecStages * kDecStageBytes <= kSmemData, "decode ring too large");
 
-// TMEM columns: S buffers [0,128) and [128,256) (fp32), O [256,384) (fp32),
-// Q [384,448) (bf16 pairs, the A operand of Q.K^T).  P_b (bf16 pairs, the A
-// operand of P.V) overwrites the first 64 columns of S_b once they are read,
-// so that both MMAs read only K or V from shared memory.
+// TMEM columns: three S buffers [0,128), [128,256), [256,384) (fp32) and O
+// [384,512) (fp32).  P_b (bf16 pairs, the A operand of P.V) overwrites the
+// first 64 columns of S_b once they are read.  Three S buffers let Q.K^T run
+// two key tiles ahead of P.V, so the softmax never waits for its scores.
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kTmemO = 256;
-constexpr uint32_t kTmemQ = 384;
+constexpr int kSBuf = 3;
+constexpr uint32_t kTmemO = kSBuf * 128;
 
 enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
 

@@ -33,19 +33,19 @@ namespace mx {
 struct Misc {
     uint64_t bar_q;
     uint64_t bar_kfull[kKStages];
-    uint64_t bar_kempty[kKStages];
-    uint64_t bar_sfull[2];
-    // P_b written (128 softmax arrivals) and V tile b landed (the V
-    // producer's arrive + transaction bytes): the one wait before P_b V_b
-    uint64_t bar_pfull[2];
-    uint64_t bar_odone[2];  // P.V of P buffer b done; frees P buffer b and V stage b
+    uint64_t bar_sfull[kSBuf];
+    // P_c written (128 softmax arrivals) and V tile c landed (the V
+    // producer's arrive + transaction bytes): the one wait before P_c V_c
+    uint64_t bar_pfull[kSBuf];
+    uint64_t bar_odone[2];  // P_c V_c done (c & 1); frees V stage c % 2
     uint32_t tmem_base;
     int32_t item_idx[2];
     int32_t abort;
     int32_t last;
 };
 static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
-static_assert(kVStages == 2, "V stage c % 2 shares the pfull and odone barriers of P buffer c & 1");
+static_assert(kVStages == 2, "V stage c % 2 is released by the odone barrier c & 1");
+static_assert(kKStages == kSBuf, "K stage c % 3 is released by the sfull barrier c % 3");
 
 // Instruction descriptors: S = Q K^T (both K-major) and O = P V (V MN-major).
 constexpr uint32_t kIdescS = idesc_bf16_f32(128, 128, false, false);
@@ -418,7 +418,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
     const int nA = (cs + kTileN - 1) / kTileN;
     const int nT = kt1 - kt0;  // key tiles of this piece: global tiles kt0 + i
     const uint32_t sbase = smem_u32(smem);
-    const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;
+    const uint32_t sQ = sbase + kSmemQ, sK = sbase + kSmemK, sV = sbase + kSmemV;
     const uint32_t bar_q = smem_u32(&misc->bar_q);
     volatile int *abort = &misc->abort;
     const uint64_t tmo = P.timeout_ns;
@@ -428,14 +428,21 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         // warp 0 loads Q and the K tiles, warp 3 the V tiles; each waits only
         // on its own ring's "empty" barriers.
         const bool isK = warp == 0;
+        if (isK && lane == 0) {
+            fence_proxy_async_smem();
+            mbar_expect_tx(bar_q, kTileBytes);
+            tma_load_3d(sQ, &P.tm_q, bar_q, 0, hq, nd + kTileM * t);
+            tma_load_3d(sQ + kHalfTile, &P.tm_q, bar_q, 64, hq, nd + kTileM * t);
+        }
         const int nst = isK ? kKStages : kVStages;
         const uint32_t ring = isK ? sK : sV;
         const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
         const void *tm_in = isK ? (const void *)&P.tm_k : (const void *)&P.tm_v;
         uint64_t *full = isK ? misc->bar_kfull : misc->bar_pfull;
-        // V stage c % 2 is free once P_{c-2} V_{c-2} has completed, which is
-        // exactly the odone barrier of P buffer c & 1 (one commit fewer per tile).
-        uint64_t *empty = isK ? misc->bar_kempty : misc->bar_odone;
+        // V stage c % 2 is free once P_{c-2} V_{c-2} has completed: the
+        // odone barrier c & 1 (one commit fewer per tile).  V_c lands on
+        // pfull c % 3, whose phase for tile c - 3 completed before that.
+        uint64_t *empty = isK ? misc->bar_sfull : misc->bar_odone;
         const int oob_row = P.num_pages * P.hkv * kPage;
         // Page ids of cached tiles, four tiles (32 pages, one per lane) per
         // load, fetched one batch ahead: a page-table read under load takes
@@ -480,7 +487,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             if (!ok)
                 break;
             if (lane == 0) {
-                const uint32_t fb = smem_u32(&full[st]);
+                const uint32_t fb = smem_u32(&full[isK ? st : (int)(c % kSBuf)]);
                 const uint32_t dst = ring + st * kTileBytes;
                 mbar_expect_tx(fb, kTileBytes);
                 if (paged) {
@@ -501,16 +508,18 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
-        // One straight loop: S_i = Q K_i^T is issued before P_{i-1} V_{i-1},
-        // so the softmax of tile i overlaps the P.V of tile i - 1.  The
-        // descriptors are formed once per tile and advanced by constants.
-        // A wait issued behind queued MMAs returns only once they have been
-        // accepted (the tensor pipe drains and refills), so each MMA group
-        // costs one such boundary and the commits are kept to a minimum.
+        // One straight loop: S_i = Q K_i^T is issued before P_{i-2} V_{i-2}
+        // (three S buffers), so the softmax of tile i - 1 and i runs while
+        // the tensor pipe works on P.V of i - 2 and S of i.  The descriptors
+        // are formed once per tile and advanced by constants.  A wait issued
+        // behind queued MMAs returns only once they have been accepted (the
+        // tensor pipe drains and refills), so each MMA group costs one such
+        // boundary and the commits are kept to a minimum.
         if (lane == 0) {
             bool ok = mbar_wait(bar_q, item_no & 1, abort, tmo);
             tc_fence_after();
-            for (int i = 0; ok && i <= nT; ++i) {
+            const uint64_t qdesc = smem_desc(sQ, 16, 1024, kSwz128);
+            for (int i = 0; ok && i < nT + 2; ++i) {
                 if (i < nT) {
                     const uint32_t c = tile0 + i;
                     const int st = c % kKStages;
@@ -520,22 +529,20 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                     }
                     tc_fence_after();
                     const uint64_t kdesc = smem_desc(sK + st * kTileBytes, 16, 1024, kSwz128);
-                    const uint32_t d = tmem + (c & 1) * 128;
+                    const uint32_t d = tmem + (c % kSBuf) * 128;
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
-                        // 16 dims: 8 columns of Q in TMEM; +32 B inside a
-                        // 64-column half of the K-major SW128 K tile
+                        // 16 dims of K-major SW128: +32 B inside a 64-column half
                         const uint64_t off = (uint64_t)(((kk >> 2) * kHalfTile + (kk & 3) * 32) >> 4);
-                        tc_mma_ts(d, tmem + kTmemQ + kk * 8, kdesc + off, kIdescS, kk > 0 ? 1u : 0u);
+                        tc_mma_ss(d, qdesc + off, kdesc + off, kIdescS, kk > 0 ? 1u : 0u);
                     }
-                    tc_commit(smem_u32(&misc->bar_sfull[c & 1]));
-                    tc_commit(smem_u32(&misc->bar_kempty[st]));
+                    tc_commit(smem_u32(&misc->bar_sfull[c % kSBuf]));  // also frees K stage st
                 }
-                if (i > 0) {
-                    const int j = i - 1;
+                if (i >= 2) {
+                    const int j = i - 2;
                     const uint32_t c = tile0 + j;
                     const int st = c % kVStages;
-                    if (!mbar_wait(smem_u32(&misc->bar_pfull[c & 1]), (c >> 1) & 1, abort, tmo)) {
+                    if (!mbar_wait(smem_u32(&misc->bar_pfull[c % kSBuf]), (c / kSBuf) & 1, abort, tmo)) {
                         ok = false;
                         break;
                     }
@@ -544,7 +551,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                         clear_uncached_rows(dv, cs - (kt0 + j) * kTileN);
                     tc_fence_after();
                     const uint64_t vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
-                    const uint32_t pa = tmem + (c & 1) * 128;  // P_c over S_c: 8 columns per 16 keys
+                    const uint32_t pa = tmem + (c % kSBuf) * 128;  // P_c over S_c: 8 columns per 16 keys
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk)  // 16 keys of MN-major V: +2 KiB
                         tc_mma_ts(tmem + kTmemO, pa + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4), kIdescO,
@@ -564,23 +571,12 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
         const float sl = P.scale_log2;
         {
-            // Q row j of head hq into TMEM lane r (zeros past the chunk's end).
-            // Piece 0 also appends this head's share of the tile's K/V: the
-            // n_rep query heads of a KV head split its 128 tokens (head r of
-            // the group takes tokens [r*128/n_rep, (r+1)*128/n_rep)), and the
-            // 32 16-byte pieces of a token's K and V rows are split between
-            // n_rep threads.  The append's loads go out with Q's, so that one
-            // memory latency covers both.
-            uint32_t qv[64];
-            const uint4 *qrow = reinterpret_cast<const uint4 *>(P.q + ((size_t)(nd + j) * P.hq + hq) * kHeadDim);
-#pragma unroll
-            for (int x = 0; x < 16; ++x) {
-                const uint4 v4 = j < p ? __ldg(qrow + x) : make_uint4(0u, 0u, 0u, 0u);
-                qv[4 * x] = v4.x;
-                qv[4 * x + 1] = v4.y;
-                qv[4 * x + 2] = v4.z;
-                qv[4 * x + 3] = v4.w;
-            }
+            // Piece 0 appends this head's share of the tile's K/V: the n_rep
+            // query heads of a KV head split its 128 tokens (head r of the
+            // group takes tokens [r*128/n_rep, (r+1)*128/n_rep)), and the 32
+            // 16-byte pieces of a token's K and V rows are split between
+            // n_rep threads; all loads are in flight at once (two rounds for
+            // n_rep = 1), while Q and the first K tile land.
             const int per = kTileM / P.n_rep, npc = 32 / P.n_rep;
             const int u = r / P.n_rep, sub = r % P.n_rep;
             const int ja = kTileM * t + (hq % P.n_rep) * per + u;   // chunk row of this thread's token
@@ -589,33 +585,24 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             int slot = -1;
             if (app)
                 slot = __ldg(P.slots + nd + ja);
-            for (int b = 0; b < npc; b += 16) {
+            for (int b = 0; app && b < npc; b += 16) {
                 uint4 av[16];
 #pragma unroll
                 for (int x = 0; x < 16; ++x) {
                     const int pc = sub * npc + b + x;   // piece: K row 0..15, V row 16..31
-                    if (app && x < npc - b)
+                    if (x < npc - b)
                         av[x] = __ldg(reinterpret_cast<const uint4 *>((pc < 16 ? P.k : P.v) + arow) + (pc & 15));
                 }
-                if (b == 0) {
-                    tmem_st32(tl + kTmemQ, *reinterpret_cast<uint32_t(*)[32]>(&qv[0]));
-                    tmem_st32(tl + kTmemQ + 32, *reinterpret_cast<uint32_t(*)[32]>(&qv[32]));
-                    tmem_wait_st();
-                    tc_fence_before();
-                    mbar_arrive(bar_q);
-                }
-                if (app && slot >= 0) {
-                    if (slot >= P.num_pages * kPage) {
-                        if (sub == 0 && b == 0)
-                            flag_error(P, ERR_SLOT);
-                    } else {
-                        const size_t dst = (((size_t)(slot / kPage) * P.hkv + kvh) * kPage + slot % kPage) * kHeadDim;
+                if (slot >= P.num_pages * kPage) {
+                    if (sub == 0 && b == 0)
+                        flag_error(P, ERR_SLOT);
+                } else if (slot >= 0) {
+                    const size_t dst = (((size_t)(slot / kPage) * P.hkv + kvh) * kPage + slot % kPage) * kHeadDim;
 #pragma unroll
-                        for (int x = 0; x < 16; ++x) {
-                            const int pc = sub * npc + b + x;
-                            if (x < npc - b)
-                                reinterpret_cast<uint4 *>((pc < 16 ? P.k_pool : P.v_pool) + dst)[pc & 15] = av[x];
-                        }
+                    for (int x = 0; x < 16; ++x) {
+                        const int pc = sub * npc + b + x;
+                        if (x < npc - b)
+                            reinterpret_cast<uint4 *>((pc < 16 ? P.k_pool : P.v_pool) + dst)[pc & 15] = av[x];
                     }
                 }
             }
@@ -624,8 +611,8 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         bool ok = true;
         for (int i = 0; i < nT; ++i) {
             const uint32_t c = tile0 + i;
-            const int sb = c & 1;
-            if (!mbar_wait(smem_u32(&misc->bar_sfull[sb]), (c >> 1) & 1, abort, tmo)) {
+            const int sb = c % kSBuf;
+            if (!mbar_wait(smem_u32(&misc->bar_sfull[sb]), (c / kSBuf) & 1, abort, tmo)) {
                 ok = false;
                 break;
             }
@@ -652,8 +639,8 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             const float m_use = rescale ? m_new : m_run;
             const float nm = -m_use;
             // P_c (the A operand of P.V) goes over the first 64 columns of
-            // S_c, whose buffer P_{c-2} held: S_c was issued after
-            // P_{c-2} V_{c-2}, so its completion covers that read too.
+            // S_c, whose buffer P_{c-3} held: S_c was issued after
+            // P_{c-3} V_{c-3}, so its completion covers that read too.
             const float rs = row_exp_store(sv, sl, nm, tl + sb * 128);
             // The O correction comes after P, when the scores are no longer
             // live, and before P_c is released to the MMA issuer.
@@ -682,11 +669,16 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             m_run = m_use;
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(smem_u32(&misc->bar_pfull[c & 1]));
+            mbar_arrive(smem_u32(&misc->bar_pfull[sb]));
         }
         if (ok) {
+            // O is complete after the last P.V.  Its odone barrier may still
+            // be one phase behind (P_{cl-2} V_{cl-2} in flight: S_cl only
+            // covers P_{cl-3} V_{cl-3}), so P_{cl-1} V_{cl-1} is awaited
+            // first; a parity wait is unambiguous only one phase ahead.
             const uint32_t cl = tile0 + nT - 1;
-            if (!mbar_wait(smem_u32(&misc->bar_odone[cl & 1]), (cl >> 1) & 1, abort, tmo))
+            if (!mbar_wait(smem_u32(&misc->bar_odone[(cl - 1) & 1]), ((cl - 1) >> 1) & 1, abort, tmo) ||
+                !mbar_wait(smem_u32(&misc->bar_odone[cl & 1]), (cl >> 1) & 1, abort, tmo))
                 ok = false;
         }
         if (!ok) {
@@ -804,19 +796,20 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     const int tid = threadIdx.x, warp = tid >> 5;
 
     if (tid == 0) {
-        mbar_init(smem_u32(&misc->bar_q), 128);
+        mbar_init(smem_u32(&misc->bar_q), 1);
         for (int b = 0; b < kKStages; ++b) {
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
-            mbar_init(smem_u32(&misc->bar_kempty[b]), 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < kSBuf; ++b) {
             mbar_init(smem_u32(&misc->bar_sfull[b]), 1);
             mbar_init(smem_u32(&misc->bar_pfull[b]), 128 + 1);
-            mbar_init(smem_u32(&misc->bar_odone[b]), 1);
         }
+        for (int b = 0; b < 2; ++b)
+            mbar_init(smem_u32(&misc->bar_odone[b]), 1);
         misc->abort = 0;
         fence_mbar_init();
         if (P.has_prefill) {
+            tma_prefetch_desc(&P.tm_q);
             tma_prefetch_desc(&P.tm_k);
             tma_prefetch_desc(&P.tm_v);
             tma_prefetch_desc(&P.tm_kpool);
