@@ -241,7 +241,8 @@ def test_prefill_pieces_deterministic_and_reusable():
     ctx.close()
 
 
-def test_iteration_independent_layers_mode_matches():
+@pytest.mark.parametrize("mode", [2])
+def test_iteration_launch_mode_matches(mode):
     """MX_OPT_PDL=2 (layer l+1 starts on the SMs layer l frees) gives the
     bit-identical outputs and KV pages of the default mode, on a plan large
     enough for a grid of every SM, over several layers."""
@@ -250,7 +251,7 @@ def test_iteration_independent_layers_mode_matches():
     ctxs = [int(c) for c in rng.integers(1500, 4000, size=48)]
     case = Case(16, ctxs, chunk_start=512, p_t=384, seed=21)
     results = {}
-    for mode in (1, 2):
+    for mode in (1, mode):
         ctx = case.make_context()
         ctx.set_option(MX_OPT_PDL, mode)
         ctx.set_option(MX_OPT_SPLIT_KEYS, 1024)   # the same plan in both modes
@@ -262,12 +263,44 @@ def test_iteration_independent_layers_mode_matches():
         assert ctx.last_plan()["n_items"] >= torch.cuda.get_device_properties(0).multi_processor_count
         results[mode] = [(d["out"].cpu().numpy(), d["k_pool"].cpu().numpy()) for d in devs]
         ctx.close()
-    for (o1, k1), (o2, k2) in zip(results[1], results[2]):
+    for (o1, k1), (o2, k2) in zip(results[1], results[mode]):
         np.testing.assert_array_equal(o1, o2)
         np.testing.assert_array_equal(k1, k2)
-    ref = case.check({"out": results[2][0][0].view(np.uint16), "k_pool": results[2][0][1].view(np.uint16),
+    ref = case.check({"out": results[mode][0][0].view(np.uint16), "k_pool": results[mode][0][1].view(np.uint16),
                       "v_pool": devs[0]["v_pool"].cpu().numpy().view(np.uint16)})
     _ok(ref)
+
+
+@pytest.mark.parametrize("mode", [1])
+def test_dependent_mode_chains_layers(mode):
+    """Dependent order: layer l+1's queries are layer l's output (the same
+    buffer), as in a model.  The default launch mode (programmatic dependent
+    launch) must give the bit-identical chain of ordinary stream order
+    (MX_OPT_PDL=0): a layer that read its queries before the previous layer
+    finished would differ."""
+    from paper_2609_38386_gb300 import MX_OPT_PDL, MX_OPT_SPLIT_KEYS
+    rng = np.random.default_rng(5)
+    ctxs = [int(c) for c in rng.integers(1000, 3000, size=40)]
+    case = Case(16, ctxs, chunk_start=256, p_t=512, seed=31)
+    n_layers = 6
+    results = {}
+    for m in (0, mode):
+        ctx = case.make_context()
+        ctx.set_option(MX_OPT_PDL, m)
+        ctx.set_option(MX_OPT_SPLIT_KEYS, 1024)
+        devs = [case.device_inputs() for _ in range(n_layers)]
+        outs = [torch.zeros_like(devs[0]["out"]) for _ in range(n_layers)]
+        # layer l+1 reads layer l's output as its q
+        qs = [devs[0]["q"]] + outs[:-1]
+        layers = [ctx.make_bufs(qs[l], devs[l]["k"], devs[l]["v"], devs[l]["k_pool"], devs[l]["v_pool"], outs[l])
+                  for l in range(n_layers)]
+        desc = case.desc(ctx, devs[0])
+        ctx.iteration(desc, layers)
+        assert ctx.last_plan()["n_items"] >= torch.cuda.get_device_properties(0).multi_processor_count
+        results[m] = [o.cpu().numpy() for o in outs] + [d["k_pool"].cpu().numpy() for d in devs]
+        ctx.close()
+    for a, b in zip(results[0], results[mode]):
+        np.testing.assert_array_equal(a, b)
 
 
 @pytest.mark.parametrize("split", [0, 512])
