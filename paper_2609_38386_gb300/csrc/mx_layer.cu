@@ -72,9 +72,23 @@ __device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t
                                                   int pid, int kb, int n, int k_hi, int di,
                                                   int h, int lane)
 {
+    const size_t pbase = ((size_t)(pid < 0 ? 0 : pid) * P.hkv + h) * kPage * kHeadDim;
+    if (pid >= 0 && kb + kPage <= n && kb + kPage <= k_hi) {
+        // a whole cached page (the common case): no per-row selection
+        const int c = lane & 15, r0 = lane >> 4;
+        const size_t off = pbase + r0 * kHeadDim + c * 8;
+        const uint16_t *ks = P.k_pool + off, *vs = P.v_pool + off;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int row = r0 + 2 * e;
+            const uint32_t dst = stage + row * 256 + ((c ^ (row & 7)) << 4);
+            cp_async16(dst, ks + 2 * e * kHeadDim, 16u);
+            cp_async16(dst + kPageBytes, vs + 2 * e * kHeadDim, 16u);
+        }
+        return;
+    }
     const uint16_t *kin = P.k + ((size_t)di * P.hkv + h) * kHeadDim;
     const uint16_t *vin = P.v + ((size_t)di * P.hkv + h) * kHeadDim;
-    const size_t pbase = ((size_t)(pid < 0 ? 0 : pid) * P.hkv + h) * kPage * kHeadDim;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
         const int ci = lane + 32 * e;  // 16-byte chunk of the 16 x 256 B page tile
@@ -198,9 +212,12 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
         const int kb = (pg_lo + warp + kWarps * k) * kPage;
         const int nv = min(kPage, k_hi - kb);  // valid keys in this page (>= 1)
 
-        // S^T (16 keys x 8 query rows) = K (16 x 128) * Q^T (128 x 8)
-        float sc[4] = {0.f, 0.f, 0.f, 0.f};
+        // S^T (16 keys x 8 query rows) = K (16 x 128) * Q^T (128 x 8), in two
+        // independent accumulation chains (even and odd 16-dim steps) so that
+        // consecutive MMAs do not wait for each other
+        float sc[4];
         {
+            float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
             const int mi = lane >> 3;
             const int row = (lane & 7) + (mi & 1) * 8;
 #pragma unroll
@@ -208,8 +225,11 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
                 const int chunk = kk * 2 + (mi >> 1);
                 uint32_t a0, a1, a2, a3;
                 ldsm_x4(kbase + row * 256 + ((chunk ^ (row & 7)) << 4), a0, a1, a2, a3);
-                mma_bf16_16816(sc, a0, a1, a2, a3, qb[kk][0], qb[kk][1]);
+                mma_bf16_16816((kk & 1) ? sb : sa, a0, a1, a2, a3, qb[kk][0], qb[kk][1]);
             }
+#pragma unroll
+            for (int x = 0; x < 4; ++x)
+                sc[x] = sa[x] + sb[x];
         }
         // online softmax over this page's keys (log2 domain), per query column
         const float x0 = g < nv ? sc[0] * sl : neg_inf();
@@ -222,21 +242,28 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
             mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
             mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
         }
+        // Lazy rescale: the running max moves (and O and l are rescaled) only
+        // when some column's max grows by more than 8 in log2 units, so p
+        // stays below 2^8; most pages skip the 32 multiplications.
         const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-        const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
-        const float p0 = ex2(x0 - mn0), p1 = ex2(x1 - mn1);
-        const float p2 = ex2(x2 - mn0), p3 = ex2(x3 - mn1);
-        l0 = l0 * al0 + p0 + p2;
-        l1 = l1 * al1 + p1 + p3;
-        m0 = mn0;
-        m1 = mn1;
+        if (__any_sync(0xffffffffu, mn0 > m0 + 8.0f || mn1 > m1 + 8.0f)) {
+            const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
+            l0 *= al0;
+            l1 *= al1;
+            m0 = mn0;
+            m1 = mn1;
 #pragma unroll
-        for (int mt = 0; mt < 8; ++mt) {
-            acc[mt][0] *= al0;
-            acc[mt][1] *= al1;
-            acc[mt][2] *= al0;
-            acc[mt][3] *= al1;
+            for (int mt = 0; mt < 8; ++mt) {
+                acc[mt][0] *= al0;
+                acc[mt][1] *= al1;
+                acc[mt][2] *= al0;
+                acc[mt][3] *= al1;
+            }
         }
+        const float p0 = ex2(x0 - m0), p1 = ex2(x1 - m1);
+        const float p2 = ex2(x2 - m0), p3 = ex2(x3 - m1);
+        l0 += p0 + p2;
+        l1 += p1 + p3;
         // P^T as the B operand (keys x query rows): transpose the 8x8 blocks
         const uint32_t b0 = movmatrix_t(pack_bf16(p0, p1));
         const uint32_t b1 = movmatrix_t(pack_bf16(p2, p3));
