@@ -32,6 +32,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
+SPEC_HBM = 8000e9          # nominal HBM3e bytes/s
+SPEC_TFLOPS = 1706.7e12   # nominal sustained dense bf16 flop/s
 METRIC = ("mixed-iteration device µs & tokens/s; % of HBM/tensor roofline per chunk size")
 UNIT = "tokens/s"
 DEFAULT_CONFIG = "qwen3-0.6b-attn-28L-chunk-sweep"
@@ -660,12 +662,19 @@ def main():
         p99 = float(np.percentile(samples, 99))
         if p == 0:
             p0_p99 = p99
+        # beside the measured peaks: the nominal 8 TB/s and 1706.7 TFLOP/s
+        # sustained, and the bound with no HBM/tensor overlap at all
+        roof_spec = sum(max(F[i] / SPEC_TFLOPS, B[i] / SPEC_HBM) for i in idx)
+        no_overlap = sum(F[i] / tfl + B[i] / hbm for i in idx)
         per_chunk[str(p)] = {
             "iterations": len(idx), "samples": int(samples.size),
             "device_us_p50": float(np.percentile(samples, 50)), "device_us_p99": p99,
             "tokens_per_s": toks / t_sum,
             "roofline_us_per_iter": roof / len(idx) * 1e6,
             "roofline_frac": roof / t_sum,
+            "roofline_frac_spec": roof_spec / t_sum,
+            "no_overlap_us_per_iter": no_overlap / len(idx) * 1e6,
+            "no_overlap_frac": no_overlap / t_sum,
             "bound": "tensor" if sum(F[idx]) / tfl > sum(B[idx]) / hbm else "hbm",
             "hbm_gbs": float(B[idx].sum() / t_sum / 1e9),
             "tflops": float(F[idx].sum() / t_sum / 1e12)}
