@@ -311,3 +311,17 @@ def test_decode_long_contexts_equal_parts(split):
     case = Case(32, [33000, 17, 4100, 513], seed=40 + split)
     res = case.run_gpu(options={MX_OPT_SPLIT_KEYS: split} if split else None)
     _ok(case.check(res))
+
+
+def test_prefix_cache_hit_shared_pages():
+    """A prefix-cache hit: the chunk's cached prefix is another sequence's
+    pages (its page-table row points at the decoding sequence's first 16
+    pages, chunk_start = 256), read by both while each appends to its own
+    pages.  Outputs within tolerance of the oracle, pages bit-exact."""
+    from synth import workload as wl
+    geom = wl.Geometry(16)
+    ctx = [300, 40]
+    layout = wl.make_layout(geom, [c + 1 for c in ctx] + [256 + 200], seed=77, spare_pages=1)
+    layout.page_table[2, :16] = layout.page_table[0, :16]
+    case = Case(16, ctx, chunk_start=256, p_t=200, seed=9, layout=layout)
+    _ok(case.check(case.run_gpu()))
