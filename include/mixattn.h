@@ -180,6 +180,15 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
  * 0: ordinary stream order.  Consecutive launches use three workspace sets
  * in turn. */
 #define MX_OPT_PDL 4
+/* MX_OPT_WAIT_LIMIT_US: bound on every in-kernel wait, in microseconds
+ * (0 = the default, one second); a wait that reaches it ends the launch with
+ * MX_ETIMEOUT.  MX_OPT_TEST_STALL_BLOCK (fault injection, 0 = off): with
+ * value b > 0, block b - 1 of every later launch claims its first work item
+ * and then waits on a barrier that nothing arrives at, so the launch reports
+ * MX_ETIMEOUT after the wait limit with that item undone.  After any
+ * reported error the context clears its counters and stays usable. */
+#define MX_OPT_WAIT_LIMIT_US 5
+#define MX_OPT_TEST_STALL_BLOCK 6
 int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 
 /* Number of work items and decode split length chosen for the last planned

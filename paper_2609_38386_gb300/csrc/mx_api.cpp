@@ -83,6 +83,9 @@ struct mx_ctx {
     int grid_opt = 0;
     int piece_tiles_opt = 0;
     int pdl = 1;  // MX_OPT_PDL: 0 stream order, 1 dependent layers, 2 independent layers
+    uint64_t wait_limit_ns = kTimeoutNs;  // MX_OPT_WAIT_LIMIT_US
+    int stall_block = -1;                 // MX_OPT_TEST_STALL_BLOCK - 1
+    size_t merge_bytes = 0, pre_cnt_bytes = 0;
     // last plan
     int last_items = 0, last_split = 0, last_prefill_items = 0, last_piece_tiles = 0;
     std::string last_error;
@@ -405,7 +408,8 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->split_keys = pl.split_keys;
     P->has_prefill = pl.n_prefill > 0 ? 1 : 0;
     P->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
-    P->timeout_ns = kTimeoutNs;
+    P->timeout_ns = c->wait_limit_ns;
+    P->stall_block = c->stall_block;
     if (P->has_prefill) {
         const cuuint64_t hd = kHeadDim;
         {
@@ -466,9 +470,18 @@ int read_error_word(mx_ctx *c)
         return cuda_fail(c, e, "reading the error word");
     if (w == 0)
         return MX_OK;
-    e = cudaMemset(c->err, 0, sizeof(uint32_t));
+    // A launch that flagged an error may have left items undone, so its
+    // arrival and work counters (normally reset by the launch itself) are
+    // cleared too; the stream has been waited on, so the workspace is idle.
+    cudaStream_t s = c->up_stream;
+    for (int k = 0; k < kWorkSets && e == cudaSuccess; ++k)
+        if ((e = cudaMemsetAsync(c->set[k].merge_cnt, 0, c->merge_bytes, s)) == cudaSuccess &&
+            (e = cudaMemsetAsync(c->set[k].pre_cnt, 0, c->pre_cnt_bytes, s)) == cudaSuccess)
+            e = cudaMemsetAsync(c->set[k].work_cnt, 0, 256, s);
+    if (e == cudaSuccess && (e = cudaMemsetAsync(c->err, 0, sizeof(uint32_t), s)) == cudaSuccess)
+        e = cudaStreamSynchronize(s);
     if (e != cudaSuccess)
-        return cuda_fail(c, e, "clearing the error word");
+        return cuda_fail(c, e, "clearing the error word and counters");
     if (w & ERR_TIMEOUT)
         return fail(c, MX_ETIMEOUT, "a bounded in-kernel wait timed out (error word 0x%x)", w);
     if (w & ERR_PAGE)
@@ -543,6 +556,8 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     const size_t pre_o_bytes = (size_t)kPrePartSlots * kTileM * kHeadDim * sizeof(float);
     const size_t pre_lse_bytes = (size_t)kPrePartSlots * kTileM * sizeof(float);
     const size_t pre_cnt_bytes = (((size_t)max_qtiles * g->num_q_heads * sizeof(uint32_t)) + 255) & ~size_t(255);
+    c->merge_bytes = merge_bytes;
+    c->pre_cnt_bytes = pre_cnt_bytes;
     c->plan_bytes = plan_capacity_bytes(c);
     const size_t plan_stride = (c->plan_bytes + 255) & ~size_t(255);
     const size_t set_bytes = part_o_bytes + part_lse_bytes + ((merge_bytes + 255) & ~size_t(255)) +
@@ -790,6 +805,16 @@ int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
         if (value < 0 || value > 65535)
             return fail(c, MX_EINVAL, "grid must be in [0, 65535]");
         c->grid_opt = (int)value;
+        return MX_OK;
+    case MX_OPT_WAIT_LIMIT_US:
+        if (value < 0 || value > 10000000)
+            return fail(c, MX_EINVAL, "wait limit must be in [0, 10^7] us");
+        c->wait_limit_ns = value == 0 ? kTimeoutNs : (uint64_t)value * 1000ull;
+        return MX_OK;
+    case MX_OPT_TEST_STALL_BLOCK:
+        if (value < 0 || value > 65535)
+            return fail(c, MX_EINVAL, "stall block must be in [0, 65535]");
+        c->stall_block = (int)value - 1;
         return MX_OK;
     default:
         return fail(c, MX_EINVAL, "unknown option %d", option);

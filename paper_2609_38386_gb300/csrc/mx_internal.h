@@ -128,6 +128,7 @@ struct LayerParams {
     int32_t early_start;   // let the next launch start as soon as this one is resident
     float scale_log2;      // log2(e) / sqrt(head_dim)
     uint64_t timeout_ns;   // bound on every in-kernel wait
+    int32_t stall_block;   // fault injection: this block's first wait never completes (-1 = none)
 };
 
 }  // namespace mx

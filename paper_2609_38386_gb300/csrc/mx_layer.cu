@@ -38,6 +38,7 @@ struct Misc {
     // producer's arrive + transaction bytes): the one wait before P_c V_c
     uint64_t bar_pfull[kSBuf];
     uint64_t bar_odone[2];  // P_c V_c done (c & 1); frees V stage c % 2
+    uint64_t bar_never;     // fault injection: a barrier nothing arrives at
     uint32_t tmem_base;
     int32_t item_idx[2];
     int32_t abort;
@@ -833,6 +834,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         }
         for (int b = 0; b < 2; ++b)
             mbar_init(smem_u32(&misc->bar_odone[b]), 1);
+        mbar_init(smem_u32(&misc->bar_never), 1);
         misc->abort = 0;
         fence_mbar_init();
         if (P.has_prefill) {
@@ -850,8 +852,15 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     // Consecutive launches use alternate workspace sets, and the launch two
     // back has completed before this one was launched (see the end of the
     // kernel), so work starts at once, beside the previous layer's tail.
-    if (tid == 0)
+    if (tid == 0) {
         misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
+        // Fault injection for the bounded waits: the chosen block waits on a
+        // barrier that nothing arrives at, with its first item claimed, so
+        // the launch ends with that item undone and its counters left set.
+        if ((int)blockIdx.x == P.stall_block &&
+            !mbar_wait(smem_u32(&misc->bar_never), 0, &misc->abort, P.timeout_ns))
+            set_abort(P, misc);
+    }
     // Independent layers (early_start): the next launch may start once every
     // CTA of this one is resident; its CTAs take the SMs this grid frees, so
     // the next layer's work fills this layer's tail.  Consecutive launches

@@ -292,6 +292,7 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     P.has_prefill = n_prefill > 0 ? 1 : 0;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     P.timeout_ns = 1000000000ull;
+    P.stall_block = -1;
     if (P.has_prefill) {
         const cuuint64_t hd = kHeadDim;
         const cuuint64_t dq[3] = {hd, (cuuint64_t)hq, (cuuint64_t)n_tok};

@@ -325,3 +325,75 @@ def test_prefix_cache_hit_shared_pages():
     layout.page_table[2, :16] = layout.page_table[0, :16]
     case = Case(16, ctx, chunk_start=256, p_t=200, seed=9, layout=layout)
     _ok(case.check(case.run_gpu()))
+
+
+@pytest.mark.parametrize("kind", ["decode_splits", "prefill_pieces"])
+def test_bounded_wait_times_out_and_context_recovers(kind):
+    """Fault injection for the bounded waits: block 0 claims its first work
+    item, then waits on a barrier that nothing arrives at.  The wait gives up
+    at the wait limit, the launch reports MX_ETIMEOUT instead of hanging, and
+    the next call on the same context is correct although the lost item left
+    its arrival counter set (a decode split's merge counter, or a prefill
+    piece's)."""
+    from paper_2609_38386_gb300 import (MX_OPT_PREFILL_PIECE_TILES, MX_OPT_SPLIT_KEYS,
+                                        MX_OPT_TEST_STALL_BLOCK, MX_OPT_WAIT_LIMIT_US, MxError)
+    if kind == "decode_splits":
+        case = Case(16, [3000, 2500, 1700, 40], seed=31)
+        opts = {MX_OPT_SPLIT_KEYS: 512}
+    else:
+        case = Case(16, [900, 40], chunk_start=700, p_t=256, seed=32)
+        opts = {MX_OPT_PREFILL_PIECE_TILES: 2}
+    ctx = case.make_context()
+    for k_, v_ in opts.items():
+        ctx.set_option(k_, v_)
+    ctx.set_option(MX_OPT_WAIT_LIMIT_US, 2000)
+    ctx.set_option(MX_OPT_TEST_STALL_BLOCK, 1)
+    with pytest.raises(MxError) as ei:
+        case.run_gpu(ctx=ctx)
+    assert "ETIMEOUT" in str(ei.value)
+    ctx.set_option(MX_OPT_TEST_STALL_BLOCK, 0)
+    ctx.set_option(MX_OPT_WAIT_LIMIT_US, 0)
+    r1 = case.run_gpu(ctx=ctx)
+    _ok(case.check(r1))
+    r2 = case.run_gpu(ctx=ctx)
+    np.testing.assert_array_equal(r1["out"], r2["out"])
+    ctx.close()
+
+
+@pytest.mark.parametrize("mode", [1, 2])
+def test_bounded_wait_timeout_in_iteration(mode):
+    """The same injected stall in every layer launch of an iteration, in both
+    launch orders: the iteration reports MX_ETIMEOUT, and the next iteration
+    on the context matches a fresh context bit for bit."""
+    from paper_2609_38386_gb300 import (MX_OPT_PDL, MX_OPT_SPLIT_KEYS, MX_OPT_TEST_STALL_BLOCK,
+                                        MX_OPT_WAIT_LIMIT_US, MxError)
+    rng = np.random.default_rng(33)
+    ctxs = [int(c) for c in rng.integers(1500, 4000, size=48)]
+    case = Case(16, ctxs, chunk_start=512, p_t=384, seed=34)
+
+    def run(ctx):
+        devs = [case.device_inputs() for _ in range(3)]
+        layers = [ctx.make_bufs(d["q"], d["k"], d["v"], d["k_pool"], d["v_pool"], d["out"]) for d in devs]
+        ctx.iteration(case.desc(ctx, devs[0]), layers)
+        torch.cuda.synchronize()
+        return [d["out"].cpu().numpy() for d in devs]
+
+    ctx = case.make_context()
+    ctx.set_option(MX_OPT_PDL, mode)
+    ctx.set_option(MX_OPT_SPLIT_KEYS, 1024)
+    ctx.set_option(MX_OPT_WAIT_LIMIT_US, 2000)
+    ctx.set_option(MX_OPT_TEST_STALL_BLOCK, 1)
+    with pytest.raises(MxError) as ei:
+        run(ctx)
+    assert "ETIMEOUT" in str(ei.value)
+    ctx.set_option(MX_OPT_TEST_STALL_BLOCK, 0)
+    ctx.set_option(MX_OPT_WAIT_LIMIT_US, 0)
+    got = run(ctx)
+    ctx.close()
+    fresh = case.make_context()
+    fresh.set_option(MX_OPT_PDL, mode)
+    fresh.set_option(MX_OPT_SPLIT_KEYS, 1024)
+    want = run(fresh)
+    fresh.close()
+    for g, w in zip(got, want):
+        np.testing.assert_array_equal(g, w)
