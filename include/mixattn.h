@@ -196,6 +196,39 @@ int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
                  int32_t *n_prefill_items);
 
+/* The work list of one layer launch, computed on the host without a device
+ * (the planning step of mx_mixed_attention / mx_iteration, exposed so that
+ * schedulers and tests can inspect it).  The paper schedules per iteration a
+ * decode set D_t and a prefill chunk of p_t tokens (§2.1, Eq. 1); one launch
+ * splits that work into items that its persistent CTAs claim in order:
+ * prefill query tiles (128 rows x one query head, or a key piece of one),
+ * heaviest first, then decode splits (one decode x one KV head x a key
+ * range), longest first.
+ *
+ * geom and desc as for mx_create / mx_mixed_attention (desc's page_table and
+ * slots are not read and may be NULL); num_sms: the SM count the launch will
+ * use; split_keys_opt, piece_tiles_opt, pdl: the values of MX_OPT_SPLIT_KEYS,
+ * MX_OPT_PREFILL_PIECE_TILES and MX_OPT_PDL (0, 0 and 1 are the defaults).
+ * Outputs (host arrays owned by the caller):
+ *   items    int32 [max_items][4], n_items records in claim order:
+ *     prefill {0, t | hq << 16, s | n_s << 16, partial slot base}: piece s
+ *       of n_s of query tile t (chunk rows [128 t, 128 t + 128)) of query
+ *       head hq; the tile's n_T = ceil(chunk_start / 128) + t + 1 key tiles
+ *       (128 keys each) are split as [s n_T / n_s, (s + 1) n_T / n_s);
+ *     decode {1 | h << 4 | s << 11 | (len / 16) << 23, decode index i,
+ *       page-table row, cached tokens ctx}: split s of decode i, KV head h,
+ *       keys [s len, min((s + 1) len, ctx + 1));
+ *   decodes  int32 [n_decodes][4]: page-table row, ctx, number of splits,
+ *     first partial slot (of head 0; head h uses base + h * splits);
+ *   counts   int32 [4]: n_items, prefill items, split_keys, piece_tiles.
+ * Returns MX_OK, MX_EINVAL (arguments, geometry, descriptor) or MX_ECAPACITY
+ * (the work does not fit max_items or the context's partial workspace), with
+ * a message in err_buf (up to err_len bytes) when err_buf is not NULL. */
+int mx_plan_work(const mx_geom *geom, const mx_iter_desc *desc, int32_t num_sms,
+                 int32_t split_keys_opt, int32_t piece_tiles_opt, int32_t pdl,
+                 int32_t *items, int32_t max_items, int32_t *decodes,
+                 int32_t *counts, char *err_buf, int32_t err_len);
+
 /* For callers that cannot allocate device memory (a host framework whose
  * allocator owns the GPU, a plug-in with a fixed pre-reserved budget, a path
  * that must not risk an allocation's implicit synchronisation or OOM).  The

@@ -28,7 +28,7 @@ MX_OPT_TEST_STALL_BLOCK = 6
 # Names every C-ABI build must export (the declarations of include/mixattn.h).
 EXPORTS = ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",
            "mx_iteration", "mx_sync_status", "mx_error_detail", "mx_set_option",
-           "mx_last_plan", "mx_mixed_attention_noalloc")
+           "mx_last_plan", "mx_plan_work", "mx_mixed_attention_noalloc")
 
 
 class MxError(RuntimeError):
@@ -80,6 +80,8 @@ def load():
             "mx_last_plan": [P, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)],
             "mx_mixed_attention_noalloc": [ctypes.POINTER(mx_geom), ctypes.POINTER(mx_iter_desc),
                                            ctypes.POINTER(mx_layer_bufs), P, ctypes.c_char_p, i32],
+            "mx_plan_work": [ctypes.POINTER(mx_geom), ctypes.POINTER(mx_iter_desc), i32, i32, i32, i32,
+                             P, i32, P, P, ctypes.c_char_p, i32],
         }
         for name, args in sig.items():
             f = getattr(lib, name)
@@ -87,6 +89,34 @@ def load():
             f.restype = ctypes.c_int
         _lib = lib
     return _lib
+
+
+def plan_work(*, num_q_heads, num_kv_heads=8, num_pages, num_seqs, max_pages_per_seq,
+              max_tokens, max_decodes, decode_seq_ids, decode_ctx_lens, prefill_seq_id=-1,
+              chunk_start=0, p_t=0, num_sms=152, split_keys=0, piece_tiles=0, pdl=1,
+              max_items=1 << 16):
+    """The work list a launch would run (host only, no device): items
+    int32 [n, 4] in claim order, decodes int32 [n_decodes, 4] and the counts
+    (n_items, prefill items, split_keys, piece_tiles)."""
+    lib = load()
+    geom = mx_geom(num_q_heads, num_kv_heads, 128, 16, num_pages, num_seqs, max_pages_per_seq,
+                   max_tokens, max_decodes)
+    ids = np.ascontiguousarray(np.asarray(decode_seq_ids, dtype=np.int32))
+    lens = np.ascontiguousarray(np.asarray(decode_ctx_lens, dtype=np.int32))
+    desc = mx_iter_desc(ids.ctypes.data if len(ids) else None, lens.ctypes.data if len(lens) else None,
+                        len(lens), int(prefill_seq_id), int(chunk_start), int(p_t), None, None)
+    items = np.zeros((max(max_items, 1), 4), np.int32)
+    decs = np.zeros((max(len(lens), 1), 4), np.int32)
+    counts = np.zeros(4, np.int32)
+    err = ctypes.create_string_buffer(512)
+    rc = lib.mx_plan_work(ctypes.byref(geom), ctypes.byref(desc), int(num_sms), int(split_keys),
+                          int(piece_tiles), int(pdl), items.ctypes.data, int(max_items),
+                          decs.ctypes.data, counts.ctypes.data, err, 512)
+    if rc != MX_OK:
+        raise MxError(rc, err.value.decode(errors="replace"))
+    return {"items": items[:counts[0]].copy(), "decodes": decs[:len(lens)].copy(),
+            "n_items": int(counts[0]), "n_prefill_items": int(counts[1]),
+            "split_keys": int(counts[2]), "piece_tiles": int(counts[3])}
 
 
 def _ptr(t):

@@ -25,6 +25,8 @@ cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int nu
 
 using namespace mx;
 
+static_assert(sizeof(DecodeInfo) == 16 && sizeof(int4) == 16, "plan records are four int32");
+
 namespace {
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
@@ -129,39 +131,76 @@ size_t plan_capacity_bytes(const mx_ctx *c)
     return (size_t)std::max(c->g.max_decodes, 1) * sizeof(DecodeInfo) + (size_t)c->max_items * sizeof(int4);
 }
 
-int validate(mx_ctx *c, const mx_iter_desc *d)
+// The geometries the kernels support.
+bool geom_ok(const mx_geom &g)
 {
-    if (!c || !d)
-        return fail(c, MX_EINVAL, "null context or descriptor");
-    const mx_geom &g = c->g;
+    if (g.head_dim != kHeadDim || g.page_size != kPage || g.num_kv_heads <= 0 ||
+        g.num_kv_heads > kMaxDecodeKvHeads || g.num_q_heads <= 0 || g.num_q_heads % g.num_kv_heads != 0 ||
+        g.num_q_heads / g.num_kv_heads > kMaxRep || g.num_pages <= 0 || g.num_seqs <= 0 ||
+        g.max_pages_per_seq <= 0 || g.max_tokens < 0 || g.max_decodes < 0 ||
+        (int64_t)g.num_pages * g.num_kv_heads * kPage > INT32_MAX)
+        return false;
+    const int rep = g.num_q_heads / g.num_kv_heads;
+    return (rep & (rep - 1)) == 0;
+}
+
+// Errors of the context-free helpers below go to a string.
+int fail_to(std::string *err, int code, const char *fmt, ...)
+{
+    if (err) {
+        char buf[512];
+        va_list ap;
+        va_start(ap, fmt);
+        vsnprintf(buf, sizeof buf, fmt, ap);
+        va_end(ap);
+        *err = buf;
+    }
+    return code;
+}
+
+// Host validation of a descriptor against the geometry.  need_tables: the
+// device page table and slots must be given (a launch); planning alone reads
+// only the host arrays.
+int validate_desc(const mx_geom &g, const mx_iter_desc *d, bool need_tables, std::string *err)
+{
+    if (!d)
+        return fail_to(err, MX_EINVAL, "null descriptor");
     if (d->n_decodes < 0 || d->p_t < 0 || d->chunk_start < 0)
-        return fail(c, MX_EINVAL, "negative n_decodes, p_t or chunk_start");
+        return fail_to(err, MX_EINVAL, "negative n_decodes, p_t or chunk_start");
     if (d->n_decodes > g.max_decodes)
-        return fail(c, MX_ECAPACITY, "n_decodes %d > max_decodes %d", d->n_decodes, g.max_decodes);
+        return fail_to(err, MX_ECAPACITY, "n_decodes %d > max_decodes %d", d->n_decodes, g.max_decodes);
     if ((int64_t)d->n_decodes + d->p_t > g.max_tokens)
-        return fail(c, MX_ECAPACITY, "n_decodes + p_t = %lld > max_tokens %d",
-                    (long long)d->n_decodes + d->p_t, g.max_tokens);
+        return fail_to(err, MX_ECAPACITY, "n_decodes + p_t = %lld > max_tokens %d",
+                       (long long)d->n_decodes + d->p_t, g.max_tokens);
     const int64_t cap = (int64_t)g.max_pages_per_seq * kPage;
     if (d->n_decodes > 0 && (!d->decode_seq_ids || !d->decode_ctx_lens))
-        return fail(c, MX_EINVAL, "decode_seq_ids / decode_ctx_lens are null");
+        return fail_to(err, MX_EINVAL, "decode_seq_ids / decode_ctx_lens are null");
     for (int i = 0; i < d->n_decodes; ++i) {
         const int s = d->decode_seq_ids[i], n = d->decode_ctx_lens[i];
         if (s < 0 || s >= g.num_seqs)
-            return fail(c, MX_EINVAL, "decode %d: seq id %d outside [0, %d)", i, s, g.num_seqs);
+            return fail_to(err, MX_EINVAL, "decode %d: seq id %d outside [0, %d)", i, s, g.num_seqs);
         if (n < 0 || (int64_t)n + 1 > cap)
-            return fail(c, MX_ECAPACITY, "decode %d: ctx %d + 1 exceeds %lld page-table slots", i, n,
-                        (long long)cap);
+            return fail_to(err, MX_ECAPACITY, "decode %d: ctx %d + 1 exceeds %lld page-table slots", i, n,
+                           (long long)cap);
     }
     if (d->p_t > 0) {
         if (d->prefill_seq_id < 0 || d->prefill_seq_id >= g.num_seqs)
-            return fail(c, MX_EINVAL, "prefill seq id %d outside [0, %d)", d->prefill_seq_id, g.num_seqs);
+            return fail_to(err, MX_EINVAL, "prefill seq id %d outside [0, %d)", d->prefill_seq_id,
+                           g.num_seqs);
         if ((int64_t)d->chunk_start + d->p_t > cap)
-            return fail(c, MX_ECAPACITY, "chunk end %lld exceeds %lld page-table slots",
-                        (long long)d->chunk_start + d->p_t, (long long)cap);
+            return fail_to(err, MX_ECAPACITY, "chunk end %lld exceeds %lld page-table slots",
+                           (long long)d->chunk_start + d->p_t, (long long)cap);
     }
-    if (d->n_decodes + d->p_t > 0 && (!d->page_table || !d->slots))
-        return fail(c, MX_EINVAL, "page_table / slots are null");
+    if (need_tables && d->n_decodes + d->p_t > 0 && (!d->page_table || !d->slots))
+        return fail_to(err, MX_EINVAL, "page_table / slots are null");
     return MX_OK;
+}
+
+int validate(mx_ctx *c, const mx_iter_desc *d)
+{
+    if (!c)
+        return MX_EINVAL;
+    return validate_desc(c->g, d, true, &c->last_error);
 }
 
 int validate_bufs(mx_ctx *c, const mx_layer_bufs *b, int n_tokens)
@@ -180,11 +219,24 @@ int validate_bufs(mx_ctx *c, const mx_layer_bufs *b, int n_tokens)
     return MX_OK;
 }
 
-// a1: the per-iteration work list.  Prefill tiles first, heaviest (latest
-// rows, most keys) first; then decode splits, longest first.
-int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
+// Tunables of the planner and what it chose.
+struct PlanKnobs {
+    int num_sms;
+    int split_keys_opt;    // 0 = automatic
+    int piece_tiles_opt;   // 0 = automatic
+    int pdl;               // launch order (MX_OPT_PDL)
+    int max_items;         // capacity of the items array
+};
+struct WorkList {
+    int n_items = 0, n_prefill = 0, split_keys = 0, piece_tiles = 0;
+};
+
+// a1: the per-iteration work list, on the host, into dec[n_decodes] and
+// items[].  Prefill tiles first, heaviest (latest rows, most keys) first;
+// then decode splits, longest first.
+int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k, DecodeInfo *dec,
+                    int4 *items, WorkList *out, std::string *err)
 {
-    const mx_geom &g = c->g;
     const int hkv = g.num_kv_heads, hq = g.num_q_heads;
     const int nd = d->n_decodes;
     int64_t total_keys = 0;
@@ -192,7 +244,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         total_keys += (int64_t)d->decode_ctx_lens[i] + 1;
     total_keys *= hkv;
 
-    int split = c->split_keys_opt;
+    int split = k.split_keys_opt;
     if (split <= 0) {
         // Each split pays a fixed start-up and merge cost, so splits are as long
         // as load balance allows: about 1.5 per SM for a decode-only iteration.
@@ -205,9 +257,9 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         double per_sm = 1.5;
         if (d->p_t > 0) {
             const int n_qt = (d->p_t + kTileM - 1) / kTileM;
-            per_sm = c->pdl == 2 ? 1.0 : std::min(3.5, std::max(1.0, 3.5 - 0.5 * (n_qt - 1)));
+            per_sm = k.pdl == 2 ? 1.0 : std::min(3.5, std::max(1.0, 3.5 - 0.5 * (n_qt - 1)));
         }
-        const int64_t target_items = std::max<int64_t>(1, (int64_t)(per_sm * c->num_sms));
+        const int64_t target_items = std::max<int64_t>(1, (int64_t)(per_sm * k.num_sms));
         int64_t s = (total_keys + target_items - 1) / target_items;
         s = (s + 127) / 128 * 128;
         split = (int)std::min<int64_t>(std::max<int64_t>(s, 512), kMaxSplitKeys);
@@ -225,20 +277,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     while (count_parts(split) > kPartSlots && split < kMaxSplitKeys)
         split = std::min(split * 2, kMaxSplitKeys);
     if (count_parts(split) > kPartSlots)
-        return fail(c, MX_ECAPACITY, "decode splits exceed the partial workspace");
-
-    // staging slot: wait until its previous upload has been consumed
-    const int slot = c->plan_next;
-    c->plan_next = (slot + 1) % kPlanSlots;
-    if (c->plan_ev_used[slot]) {
-        cudaError_t e = cudaEventSynchronize(c->plan_ev[slot]);
-        if (e != cudaSuccess)
-            return cuda_fail(c, e, "cudaEventSynchronize(plan)");
-    }
-    uint8_t *host = c->plan_host[slot];
-    DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(host);
-    const size_t items_off = (size_t)nd * sizeof(DecodeInfo);
-    int4 *items = reinterpret_cast<int4 *>(host + items_off);
+        return fail_to(err, MX_ECAPACITY, "decode splits exceed the partial workspace");
 
     // Prefill tiles, split along their key tiles into pieces of at most
     // piece_tiles tiles so that long causal rows spread over several SMs.
@@ -251,12 +290,12 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     // Splitting costs a partial write and a merge; it pays only when the
     // chunk has too few tiles to occupy the GPU (short chunks deep into a
     // long prompt), so tiles are split only then, into >= 48-tile pieces.
-    int piece = c->piece_tiles_opt;
+    int piece = k.piece_tiles_opt;
     if (piece <= 0) {
-        if ((int64_t)n_qt * hq * 2 >= c->num_sms)
+        if ((int64_t)n_qt * hq * 2 >= k.num_sms)
             piece = 65535;
         else
-            piece = (int)std::max<int64_t>(kMinPieceTiles, (pre_work + c->num_sms - 1) / c->num_sms);
+            piece = (int)std::max<int64_t>(kMinPieceTiles, (pre_work + k.num_sms - 1) / k.num_sms);
     }
     auto count_pre_parts = [&](int pc) {
         int64_t parts = 0;
@@ -288,8 +327,8 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     }
     std::stable_sort(pitems.begin(), pitems.end(),
                      [](const PItem &a, const PItem &b) { return a.tiles > b.tiles; });
-    if ((int64_t)pitems.size() > c->max_items)
-        return fail(c, MX_ECAPACITY, "%zu prefill items exceed capacity %d", pitems.size(), c->max_items);
+    if ((int64_t)pitems.size() > k.max_items)
+        return fail_to(err, MX_ECAPACITY, "%zu prefill items exceed capacity %d", pitems.size(), k.max_items);
     for (const PItem &x : pitems)
         items[n++] = x.code;
     const int n_prefill = n;
@@ -306,7 +345,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         const int ns = (keys + split - 1) / split;
         const int len = ((keys + ns - 1) / ns + kPage - 1) / kPage * kPage;
         if (ns > kMaxDecodeSplits)
-            return fail(c, MX_ECAPACITY, "decode %d needs %d splits (limit %d)", i, ns, kMaxDecodeSplits);
+            return fail_to(err, MX_ECAPACITY, "decode %d needs %d splits (limit %d)", i, ns, kMaxDecodeSplits);
         dec[i].seq = d->decode_seq_ids[i];
         dec[i].ctx = d->decode_ctx_lens[i];
         dec[i].n_splits = ns;
@@ -317,13 +356,42 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
             for (int s = 0; s < ns; ++s)
                 ditems.push_back({std::min(len, keys - s * len), i, h, s, len});
     }
-    if (n_prefill + (int)ditems.size() > c->max_items)
-        return fail(c, MX_ECAPACITY, "work list of %zu items exceeds capacity %d",
-                    n_prefill + ditems.size(), c->max_items);
+    if (n_prefill + (int)ditems.size() > k.max_items)
+        return fail_to(err, MX_ECAPACITY, "work list of %zu items exceeds capacity %d",
+                       n_prefill + ditems.size(), k.max_items);
     std::stable_sort(ditems.begin(), ditems.end(),
                      [](const DItem &a, const DItem &b) { return a.keys > b.keys; });
     for (const DItem &x : ditems)
         items[n++] = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx, x.len);
+
+    out->n_items = n;
+    out->n_prefill = n_prefill;
+    out->split_keys = split;
+    out->piece_tiles = piece;
+    return MX_OK;
+}
+
+// Plans into the next pinned staging slot and uploads it.
+int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
+{
+    // staging slot: wait until its previous upload has been consumed
+    const int slot = c->plan_next;
+    c->plan_next = (slot + 1) % kPlanSlots;
+    if (c->plan_ev_used[slot]) {
+        cudaError_t e = cudaEventSynchronize(c->plan_ev[slot]);
+        if (e != cudaSuccess)
+            return cuda_fail(c, e, "cudaEventSynchronize(plan)");
+    }
+    uint8_t *host = c->plan_host[slot];
+    DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(host);
+    const size_t items_off = (size_t)d->n_decodes * sizeof(DecodeInfo);
+    int4 *items = reinterpret_cast<int4 *>(host + items_off);
+    const PlanKnobs knobs{c->num_sms, c->split_keys_opt, c->piece_tiles_opt, c->pdl, c->max_items};
+    WorkList wl;
+    int rc = build_work_list(c->g, d, knobs, dec, items, &wl, &c->last_error);
+    if (rc)
+        return rc;
+    const int n = wl.n_items;
 
     const size_t bytes = items_off + (size_t)n * sizeof(int4);
     // A kernel, not a copy engine, moves the plan (an H2D memcpy would queue
@@ -345,15 +413,15 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
         return cuda_fail(c, e, "cudaStreamWaitEvent(plan)");
 
     out->n_items = n;
-    out->n_prefill = n_prefill;
-    out->split_keys = split;
+    out->n_prefill = wl.n_prefill;
+    out->split_keys = wl.split_keys;
     out->slot = slot;
     out->items_dev = reinterpret_cast<const int4 *>(c->plan_dev[slot] + items_off);
     out->dec_dev = reinterpret_cast<const DecodeInfo *>(c->plan_dev[slot]);
     c->last_items = n;
-    c->last_split = split;
-    c->last_prefill_items = n_prefill;
-    c->last_piece_tiles = piece;
+    c->last_split = wl.split_keys;
+    c->last_prefill_items = wl.n_prefill;
+    c->last_piece_tiles = wl.piece_tiles;
     return MX_OK;
 }
 
@@ -514,15 +582,7 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     if (!out || !g)
         return MX_EINVAL;
     *out = nullptr;
-    if (g->head_dim != kHeadDim || g->page_size != kPage || g->num_kv_heads <= 0 ||
-        g->num_kv_heads > kMaxDecodeKvHeads ||
-        g->num_q_heads <= 0 || g->num_q_heads % g->num_kv_heads != 0 ||
-        g->num_q_heads / g->num_kv_heads > kMaxRep || g->num_pages <= 0 || g->num_seqs <= 0 ||
-        g->max_pages_per_seq <= 0 || g->max_tokens < 0 || g->max_decodes < 0 ||
-        (int64_t)g->num_pages * g->num_kv_heads * kPage > INT32_MAX)
-        return MX_EINVAL;
-    const int rep = g->num_q_heads / g->num_kv_heads;
-    if (rep & (rep - 1))
+    if (!geom_ok(*g))
         return MX_EINVAL;
     int ndev = 0;
     if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev)
@@ -819,6 +879,44 @@ int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
     default:
         return fail(c, MX_EINVAL, "unknown option %d", option);
     }
+}
+
+int mx_plan_work(const mx_geom *geom, const mx_iter_desc *desc, int32_t num_sms, int32_t split_keys_opt,
+                 int32_t piece_tiles_opt, int32_t pdl, int32_t *items, int32_t max_items, int32_t *decodes,
+                 int32_t *counts, char *err_buf, int32_t err_len)
+{
+    std::string err;
+    int rc = MX_OK;
+    if (!geom || !desc || !counts || (!items && max_items > 0) || max_items < 0 || num_sms <= 0 ||
+        pdl < 0 || pdl > 2 || split_keys_opt < 0 || split_keys_opt > kMaxSplitKeys || split_keys_opt % 128 ||
+        piece_tiles_opt < 0 || piece_tiles_opt > 65535)
+        rc = fail_to(&err, MX_EINVAL, "null argument or option out of range");
+    else if (!geom_ok(*geom))
+        rc = fail_to(&err, MX_EINVAL, "unsupported geometry");
+    else if ((rc = validate_desc(*geom, desc, false, &err)) == MX_OK && desc->n_decodes > 0 && !decodes)
+        rc = fail_to(&err, MX_EINVAL, "decodes is null");
+    if (rc == MX_OK) {
+        std::vector<DecodeInfo> dec((size_t)std::max(desc->n_decodes, 1));
+        std::vector<int4> it((size_t)std::max(max_items, 1));
+        const PlanKnobs knobs{num_sms, split_keys_opt, piece_tiles_opt, pdl, max_items};
+        WorkList wl;
+        rc = build_work_list(*geom, desc, knobs, dec.data(), it.data(), &wl, &err);
+        if (rc == MX_OK) {
+            std::memcpy(items, it.data(), (size_t)wl.n_items * sizeof(int4));
+            if (desc->n_decodes > 0)
+                std::memcpy(decodes, dec.data(), (size_t)desc->n_decodes * sizeof(DecodeInfo));
+            counts[0] = wl.n_items;
+            counts[1] = wl.n_prefill;
+            counts[2] = wl.split_keys;
+            counts[3] = wl.piece_tiles;
+        }
+    }
+    if (rc != MX_OK && err_buf && err_len > 0) {
+        const size_t n = std::min<size_t>(err.size(), (size_t)err_len - 1);
+        std::memcpy(err_buf, err.data(), n);
+        err_buf[n] = '\0';
+    }
+    return rc;
 }
 
 int mx_last_plan(mx_ctx *c, int32_t *n_items, int32_t *split_keys, int32_t *n_prefill_items)
