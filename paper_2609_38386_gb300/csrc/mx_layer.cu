@@ -71,7 +71,7 @@ __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000);
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t stage,
                                                   int pid, int kb, int n, int k_hi, int di,
-                                                  int h, int lane)
+                                                  int h, int lane, uint64_t pol)
 {
     const size_t pbase = ((size_t)(pid < 0 ? 0 : pid) * P.hkv + h) * kPage * kHeadDim;
     if (pid >= 0 && kb + kPage <= n && kb + kPage <= k_hi) {
@@ -83,8 +83,8 @@ __device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t
         for (int e = 0; e < 8; ++e) {
             const int row = r0 + 2 * e;
             const uint32_t dst = stage + row * 256 + ((c ^ (row & 7)) << 4);
-            cp_async16(dst, ks + 2 * e * kHeadDim, 16u);
-            cp_async16(dst + kPageBytes, vs + 2 * e * kHeadDim, 16u);
+            cp_async16_hint(dst, ks + 2 * e * kHeadDim, 16u, pol);
+            cp_async16_hint(dst + kPageBytes, vs + 2 * e * kHeadDim, 16u, pol);
         }
         return;
     }
@@ -109,8 +109,8 @@ __device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t
                 bytes = 0;
         }
         const uint32_t dst = stage + row * 256 + ((c ^ (row & 7)) << 4);
-        cp_async16(dst, ks, bytes);
-        cp_async16(dst + kPageBytes, vs, bytes);
+        cp_async16_hint(dst, ks, bytes, pol);
+        cp_async16_hint(dst + kPageBytes, vs, bytes, pol);
     }
 }
 
@@ -180,6 +180,9 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
     }
 
     const uint32_t ring = smem_u32(smem) + warp * (kDecStages * kDecStageBytes);
+    // the pages stream through once: evict_first keeps them from displacing
+    // the prefill's K/V tiles, which several query heads and tiles re-read
+    const uint64_t pol = l2_policy_evict_first();
     float acc[8][4];
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt)
@@ -192,7 +195,7 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
         const int pid = __shfl_sync(0xffffffffu, pid_l, k & 31);
         if (k < my_n)
             decode_issue_page(P, ring + k * kDecStageBytes, pid,
-                              (pg_lo + warp + kWarps * k) * kPage, n, k_hi, di, h, lane);
+                              (pg_lo + warp + kWarps * k) * kPage, n, k_hi, di, h, lane, pol);
         cp_async_commit();
     }
 
@@ -202,7 +205,7 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
             const int pid = __shfl_sync(0xffffffffu, pid_l, kn & 31);
             if (kn < my_n)
                 decode_issue_page(P, ring + (kn % kDecStages) * kDecStageBytes, pid,
-                                  (pg_lo + warp + kWarps * kn) * kPage, n, k_hi, di, h, lane);
+                                  (pg_lo + warp + kWarps * kn) * kPage, n, k_hi, di, h, lane, pol);
             cp_async_commit();
         }
         cp_async_wait<kDecStages - 1>();
