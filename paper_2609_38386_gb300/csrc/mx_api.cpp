@@ -250,14 +250,15 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
         // as load balance allows: about 1.5 per SM for a decode-only iteration.
         // Beside prefill tiles, which hold SMs from the start, the decode
         // splits must fill around them: the fewer the query tiles, the finer
-        // (3 per SM beside 2 tiles, 2 beside 4, 1 from 6 on; a sweep of
-        // 1024-4096-key splits over the 0.6B sweep's chunk sizes put the
-        // optimum there).  With independent layers (MX_OPT_PDL = 2) the next
-        // layer fills the tail, so the splits stay long.
+        // (3.5 per SM beside one tile, 3 beside 2, 2 beside 3, 1 from 4 on; a
+        // sweep of 1024-4096-key splits over the 0.6B sweep's chunk sizes put
+        // the optimum there).  With independent layers (MX_OPT_PDL = 2) the
+        // next layer fills the tail, so the splits stay long.
         double per_sm = 1.5;
         if (d->p_t > 0) {
             const int n_qt = (d->p_t + kTileM - 1) / kTileM;
-            per_sm = k.pdl == 2 ? 1.0 : std::min(3.5, std::max(1.0, 3.5 - 0.5 * (n_qt - 1)));
+            static const double kBeside[3] = {3.5, 3.0, 2.0};
+            per_sm = k.pdl == 2 ? 1.0 : (n_qt <= 3 ? kBeside[n_qt - 1] : 1.0);
         }
         const int64_t target_items = std::max<int64_t>(1, (int64_t)(per_sm * k.num_sms));
         int64_t s = (total_keys + target_items - 1) / target_items;
