@@ -55,9 +55,10 @@ struct mx_ctx {
     int max_items = 0;
     // workspace (device)
     uint8_t *ws = nullptr;
-    // Two workspace sets, used by alternate launches: a layer kernel may
-    // start while the previous one drains (programmatic dependent launch),
-    // and the one before that has completed by then.
+    // kWorkSets workspace sets, used by consecutive launches in turn: a layer
+    // kernel may start while the previous one drains (programmatic dependent
+    // launch), and by the time a set comes round again, the launch that last
+    // used it has completed.
     struct Set {
         float *part_o, *part_lse;
         uint32_t *merge_cnt;
@@ -903,7 +904,8 @@ int mx_plan_work(const mx_geom *geom, const mx_iter_desc *desc, int32_t num_sms,
         WorkList wl;
         rc = build_work_list(*geom, desc, knobs, dec.data(), it.data(), &wl, &err);
         if (rc == MX_OK) {
-            std::memcpy(items, it.data(), (size_t)wl.n_items * sizeof(int4));
+            if (wl.n_items > 0)
+                std::memcpy(items, it.data(), (size_t)wl.n_items * sizeof(int4));
             if (desc->n_decodes > 0)
                 std::memcpy(decodes, dec.data(), (size_t)desc->n_decodes * sizeof(DecodeInfo));
             counts[0] = wl.n_items;
