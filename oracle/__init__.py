@@ -47,7 +47,7 @@ def _load():
         lib.oracle_kv_append.argtypes = [P, P, i64, i32, i32, i32, P, i32, P, P]
         lib.oracle_mixed_attention.restype = ctypes.c_int
         lib.oracle_mixed_attention.argtypes = (
-            [i32, i32, i32, i32, i64, i32, P, P, i32, i32, i32, i32]
+            [i32, i32, i32, i32, i64, i32, P, P, i32, P, P, P, i32]
             + [P] * 7 + [P, i32, P, P, P, i64])
         lib.oracle_max_threads.restype = ctypes.c_int
         _lib = lib
@@ -92,13 +92,15 @@ def kv_append(k_pool, v_pool, slots, k, v, page_size=16):
 
 def mixed_attention(*, q, k, v, k_pool, v_pool, page_table, slots,
                     decode_seq_ids, decode_ctx_lens, prefill_seq=-1,
-                    chunk_start=0, p_t=0, rows=None):
+                    chunk_start=0, p_t=0, prefills=None, rows=None):
     """One layer of the mixed iteration in float64 (pools are modified).
 
-    q: uint16 [n_decodes + p_t][hq][head_dim]; k, v: uint16
-    [n_decodes + p_t][hkv][head_dim]; pools: uint16
-    [num_pages][hkv][page_size][head_dim]; page_table: int32
-    [num_seqs][max_pages]; slots: int32 [n_decodes + p_t].
+    One prefill chunk (prefill_seq, chunk_start, p_t), or several given as
+    ``prefills`` = [(seq, chunk_start, p_t), ...] (then p_t must be 0).
+    q: uint16 [n_tokens][hq][head_dim]; k, v: uint16
+    [n_tokens][hkv][head_dim] with n_tokens = n_decodes + the chunk rows;
+    pools: uint16 [num_pages][hkv][page_size][head_dim]; page_table: int32
+    [num_seqs][max_pages]; slots: int32 [n_tokens].
     Returns (out float64 [n_rows][hq][head_dim], lse float64 [n_rows][hq])
     for the requested token rows (all rows when ``rows`` is None).
     """
@@ -108,7 +110,14 @@ def mixed_attention(*, q, k, v, k_pool, v_pool, page_table, slots,
     n_tok, hq, hd2 = q.shape
     assert hd2 == hd and k.shape == (n_tok, hkv, hd) and v.shape == k.shape
     nd = len(decode_ctx_lens)
-    assert n_tok == nd + p_t
+    if prefills is None:
+        prefills = [(prefill_seq, chunk_start, p_t)] if p_t > 0 else []
+    else:
+        assert p_t == 0
+    pf_seq = _i32([pf[0] for pf in prefills] or [0])
+    pf_cs = _i32([pf[1] for pf in prefills] or [0])
+    pf_p = _i32([pf[2] for pf in prefills] or [0])
+    assert n_tok == nd + sum(pf[2] for pf in prefills)
     page_table = _i32(page_table)
     slots = _i32(slots)
     dids, dlens = _i32(decode_seq_ids), _i32(decode_ctx_lens)
@@ -116,12 +125,12 @@ def mixed_attention(*, q, k, v, k_pool, v_pool, page_table, slots,
     n_rows = n_tok if rows_a is None else len(rows_a)
     out = np.zeros((n_rows, hq, hd), dtype=np.float64)
     lse = np.zeros((n_rows, hq), dtype=np.float64)
-    max_keys = max([int(x) + 1 for x in dlens] + [chunk_start + p_t, 1])
+    max_keys = max([int(x) + 1 for x in dlens] + [pf[1] + pf[2] for pf in prefills] + [1])
     nthr = max_threads()
     scratch = np.zeros(nthr * max_keys, dtype=np.float64)
     rc = _load().oracle_mixed_attention(
         hq, hkv, hd, ps, num_pages, page_table.shape[1], _p(dids), _p(dlens),
-        nd, prefill_seq, chunk_start, p_t, _p(page_table), _p(slots), _p(q),
+        nd, _p(pf_seq), _p(pf_cs), _p(pf_p), len(prefills), _p(page_table), _p(slots), _p(q),
         _p(k), _p(v), _p(k_pool), _p(v_pool), _p(rows_a), n_rows, _p(out),
         _p(lse), _p(scratch), max_keys)
     if rc != 0:

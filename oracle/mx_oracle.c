@@ -130,8 +130,11 @@ static int attend_one(const uint16_t *qv, int n_keys, const int32_t *pt_row,
 
 /*
  * One layer of the mixed iteration (§2.1): |D_t| = n_decodes decode queries
- * and a prefill chunk of p_t rows of sequence prefill_seq starting at
- * chunk_start.  Token order in q/k/v/slots: the decodes first, then the chunk.
+ * and n_prefills prefill chunks; chunk j has p_ts[j] rows of sequence
+ * prefill_seqs[j] starting at position chunk_starts[j] (one chunk is the
+ * paper's setting; §4.1's scheduler may admit the chunks of several prompts
+ * under one token budget, each still a chunk of its own sequence).  Token
+ * order in q/k/v/slots: the decodes first, then chunk 0's rows, chunk 1's, ...
  *
  * Step 1 applies the append of all n_decodes + p_t tokens to the pools (which
  * the caller passes as its own host copies; they are modified).  Step 2
@@ -145,7 +148,8 @@ int oracle_mixed_attention(int hq, int hkv, int head_dim, int page_size,
                            int64_t num_pages, int max_pages,
                            const int32_t *decode_seq_ids,
                            const int32_t *decode_ctx_lens, int n_decodes,
-                           int prefill_seq, int chunk_start, int p_t,
+                           const int32_t *prefill_seqs, const int32_t *chunk_starts,
+                           const int32_t *p_ts, int n_prefills,
                            const int32_t *page_table, const int32_t *slots,
                            const uint16_t *q, const uint16_t *k,
                            const uint16_t *v, uint16_t *k_pool,
@@ -154,9 +158,14 @@ int oracle_mixed_attention(int hq, int hkv, int head_dim, int page_size,
                            int64_t scratch_per_thread)
 {
     if (hq <= 0 || hkv <= 0 || hq % hkv != 0 || head_dim <= 0 ||
-        page_size <= 0 || n_decodes < 0 || p_t < 0 || chunk_start < 0)
+        page_size <= 0 || n_decodes < 0 || n_prefills < 0)
         return ORC_EINVAL;
-    int n_tok = n_decodes + p_t;
+    int n_tok = n_decodes;
+    for (int j = 0; j < n_prefills; ++j) {
+        if (p_ts[j] < 0 || chunk_starts[j] < 0)
+            return ORC_EINVAL;
+        n_tok += p_ts[j];
+    }
     int rc = oracle_kv_append(k_pool, v_pool, num_pages, hkv, page_size,
                               head_dim, slots, n_tok, k, v);
     if (rc != ORC_OK)
@@ -177,8 +186,14 @@ int oracle_mixed_attention(int hq, int hkv, int head_dim, int page_size,
             seq = decode_seq_ids[r];
             n_keys = decode_ctx_lens[r] + 1;
         } else {
-            seq = prefill_seq;
-            n_keys = chunk_start + (r - n_decodes) + 1;
+            /* the chunk holding token r, and r's row within it */
+            int j = 0, row = r - n_decodes;
+            while (row >= p_ts[j]) {
+                row -= p_ts[j];
+                ++j;
+            }
+            seq = prefill_seqs[j];
+            n_keys = chunk_starts[j] + row + 1;
         }
         if (n_keys > scratch_per_thread) {
             err = ORC_EINVAL;

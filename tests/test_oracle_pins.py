@@ -40,13 +40,19 @@ class Case:
     """
 
     def __init__(self, rng, hq, hkv, d, ps, ctx, chunk_start=0, p_t=0,
-                 prompt_len=None, spare=3, perm_seed=7, q_zero=False):
+                 prompt_len=None, spare=3, perm_seed=7, q_zero=False, prefills=None):
+        # prefills: [(chunk_start, p_t, prompt_len or None), ...], one
+        # sequence each (rows nd, nd + 1, ... of the page table); the
+        # chunk_start / p_t / prompt_len arguments give a single one
         self.hq, self.hkv, self.d, self.ps = hq, hkv, d, ps
         nd = len(ctx)
         caps = [c + 1 for c in ctx]
-        self.prefill = p_t > 0
-        if self.prefill:
-            caps.append(prompt_len or chunk_start + p_t)
+        self.multi = prefills is not None
+        if prefills is None:
+            prefills = [(chunk_start, p_t, prompt_len)] if p_t > 0 else []
+        self.prefills = [(cs_, p_, pl_ or cs_ + p_) for cs_, p_, pl_ in prefills]
+        self.prefill = len(self.prefills) > 0
+        caps += [pl_ for _, _, pl_ in self.prefills]
         self.caps = caps
         self.dense_k = [_randn_bf16(rng, (c, hkv, d)) for c in caps]
         self.dense_v = [_randn_bf16(rng, (c, hkv, d)) for c in caps]
@@ -64,7 +70,7 @@ class Case:
         self.v_pool = _randn_bf16(rng, (self.num_pages, hkv, ps, d), 3.0)
         # cached positions: scatter dense contents; appended ones stay garbage
         for s, cap in enumerate(caps):
-            cached = ctx[s] if s < nd else chunk_start
+            cached = ctx[s] if s < nd else self.prefills[s - nd][0]
             for pos in range(cached):
                 pg, off = self.pt[s, pos // ps], pos % ps
                 self.k_pool[pg, :, off, :] = self.dense_k[s][pos]
@@ -79,13 +85,14 @@ class Case:
             rows_v.append(self.dense_v[i][ctx[i]])
             slots.append(self.pt[i, ctx[i] // ps] * ps + ctx[i] % ps)
             pos_of.append((i, ctx[i]))
-        for j in range(p_t):
-            pos = chunk_start + j
-            rows_k.append(self.dense_k[nd][pos])
-            rows_v.append(self.dense_v[nd][pos])
-            slots.append(self.pt[nd, pos // ps] * ps + pos % ps)
-            pos_of.append((nd, pos))
-        n_tok = nd + p_t
+        for f, (cs_, p_, _) in enumerate(self.prefills):
+            for j in range(p_):
+                pos = cs_ + j
+                rows_k.append(self.dense_k[nd + f][pos])
+                rows_v.append(self.dense_v[nd + f][pos])
+                slots.append(self.pt[nd + f, pos // ps] * ps + pos % ps)
+                pos_of.append((nd + f, pos))
+        n_tok = len(pos_of)
         self.k = np.array(rows_k, np.uint16).reshape(n_tok, hkv, d)
         self.v = np.array(rows_v, np.uint16).reshape(n_tok, hkv, d)
         self.slots = np.array(slots, np.int32)
@@ -96,6 +103,14 @@ class Case:
     def run(self, rows=None, k_pool=None, v_pool=None, pt=None):
         kp = (self.k_pool if k_pool is None else k_pool).copy()
         vp = (self.v_pool if v_pool is None else v_pool).copy()
+        if self.multi:
+            nd = len(self.ctx)
+            return oracle.mixed_attention(
+                q=self.q, k=self.k, v=self.v, k_pool=kp, v_pool=vp,
+                page_table=self.pt if pt is None else pt, slots=self.slots,
+                decode_seq_ids=self.dids, decode_ctx_lens=self.ctx,
+                prefills=[(nd + f, cs_, p_) for f, (cs_, p_, _) in enumerate(self.prefills)],
+                rows=rows)
         return oracle.mixed_attention(
             q=self.q, k=self.k, v=self.v, k_pool=kp, v_pool=vp,
             page_table=self.pt if pt is None else pt, slots=self.slots,
@@ -146,6 +161,44 @@ def test_oracle_equals_dense_bruteforce(hq, hkv, d, ps):
     want = c.brute()
     np.testing.assert_allclose(out, want, rtol=0, atol=1e-12)
     assert np.all(np.isfinite(lse))
+
+
+@pytest.mark.parametrize("hq,hkv,d,ps", [(2, 1, 8, 4), (4, 2, 128, 16)])
+def test_several_prefill_chunks_equal_dense_bruteforce(hq, hkv, d, ps):
+    """Several prompts' chunks in one iteration (each a chunk of its own
+    sequence, rows laid out one chunk after another): every row against
+    dense attention over its own sequence's keys, including a chunk at
+    position 0 and ragged lengths."""
+    rng = np.random.default_rng(hq * 7 + d + ps)
+    c = Case(rng, hq, hkv, d, ps, ctx=[0, 21],
+             prefills=[(13, 11, 30), (0, 5, None), (40, 1, 41), (3, 9, 20)])
+    out, lse = c.run()
+    np.testing.assert_allclose(out, c.brute(), rtol=0, atol=1e-12)
+    assert np.all(np.isfinite(lse))
+
+
+def test_several_prefill_chunks_one_at_a_time_bit_identical():
+    """Each chunk's rows equal, bit for bit, the rows of an iteration that
+    carries that chunk alone: chunks of different sequences do not interact
+    (a wrong row-to-chunk mapping or token offset would break this)."""
+    rng = np.random.default_rng(11)
+    pfs = [(5, 7, 20), (0, 3, None), (17, 6, 23)]
+    c = Case(rng, 4, 2, 16, 4, ctx=[3, 9], prefills=pfs)
+    full, lse_full = c.run()
+    nd = 2
+    base = nd
+    for f, (cs_, p_, _) in enumerate(pfs):
+        rows = list(range(base, base + p_))
+        kp, vp = c.k_pool.copy(), c.v_pool.copy()
+        sel = list(range(nd)) + rows
+        one, lse_one = oracle.mixed_attention(
+            q=c.q[sel], k=c.k[sel], v=c.v[sel], k_pool=kp, v_pool=vp, page_table=c.pt,
+            slots=c.slots[sel], decode_seq_ids=c.dids, decode_ctx_lens=c.ctx,
+            prefill_seq=nd + f, chunk_start=cs_, p_t=p_)
+        np.testing.assert_array_equal(full[rows], one[nd:])
+        np.testing.assert_array_equal(lse_full[rows], lse_one[nd:])
+        np.testing.assert_array_equal(full[:nd], one[:nd])
+        base += p_
 
 
 def test_oracle_rows_subset_equals_full():
