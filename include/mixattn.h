@@ -83,6 +83,17 @@ typedef struct {
     int32_t max_decodes;       /* max n_decodes per call                  */
 } mx_geom;
 
+/* One prefill chunk: positions [chunk_start, chunk_start + p_t) of the
+ * prompt in page-table row seq_id; its row j attends keys [0, chunk_start + j]
+ * of that sequence. */
+typedef struct {
+    int32_t seq_id;       /* page-table row                                 */
+    int32_t chunk_start;  /* first position of the chunk                    */
+    int32_t p_t;          /* chunk length, >= 1                             */
+} mx_prefill;
+
+#define MX_MAX_PREFILLS 16
+
 /* What one iteration schedules (§2.1: the decode set D_t and the prefill
  * budget p_t; §3.1 caps p_t).  decode_seq_ids / decode_ctx_lens are HOST
  * arrays of n_decodes entries: the page-table row of each decoding sequence
@@ -99,7 +110,15 @@ typedef struct {
     int32_t chunk_start;            /* first position of the chunk        */
     int32_t p_t;                    /* chunk length, 0 = decode only      */
     const int32_t *page_table;      /* device [num_seqs][max_pages_per_seq] */
-    const int32_t *slots;           /* device [n_decodes + p_t]           */
+    const int32_t *slots;           /* device [n_tokens]                  */
+    /* Several chunks (§4.1: the scheduler may admit chunks of several
+     * prompts under one token budget): n_prefills > 0 chunks in prefills
+     * (a HOST array), used instead of prefill_seq_id / chunk_start / p_t,
+     * which must then be -1 / 0 / 0.  At most MX_MAX_PREFILLS; their rows
+     * follow the decode tokens chunk after chunk, so n_tokens = n_decodes +
+     * the sum of their p_t.  0: the single chunk above (or none). */
+    int32_t n_prefills;
+    const mx_prefill *prefills;
 } mx_iter_desc;
 
 /* Per-layer tensors of one iteration (all DEVICE pointers). */
@@ -236,7 +255,8 @@ int mx_plan_work(const mx_geom *geom, const mx_iter_desc *desc, int32_t num_sms,
  * mx_mixed_attention that needs no context, because mx_create allocates.
  *
  * Same operation, layouts and descriptor as mx_mixed_attention (geom gives
- * the geometry a context would hold; max_tokens / max_decodes are ignored).
+ * the geometry a context would hold; max_tokens / max_decodes are ignored),
+ * for at most one prefill chunk (desc->n_prefills must be 0).
  * Its scratch (work list, split partials, counters, error word) is one fixed
  * 4.11 MiB device array built into the library, which every GPU that loads
  * the library holds until the process exits.  Limits: n_decodes <= 256,

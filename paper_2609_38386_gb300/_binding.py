@@ -43,11 +43,24 @@ class mx_geom(ctypes.Structure):
         "num_seqs", "max_pages_per_seq", "max_tokens", "max_decodes")]
 
 
+class mx_prefill(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("seq_id", "chunk_start", "p_t")]
+
+
 class mx_iter_desc(ctypes.Structure):
     _fields_ = [("decode_seq_ids", ctypes.c_void_p), ("decode_ctx_lens", ctypes.c_void_p),
                 ("n_decodes", ctypes.c_int32), ("prefill_seq_id", ctypes.c_int32),
                 ("chunk_start", ctypes.c_int32), ("p_t", ctypes.c_int32),
-                ("page_table", ctypes.c_void_p), ("slots", ctypes.c_void_p)]
+                ("page_table", ctypes.c_void_p), ("slots", ctypes.c_void_p),
+                ("n_prefills", ctypes.c_int32), ("prefills", ctypes.c_void_p)]
+
+
+def _prefill_array(prefills):
+    """[(seq, chunk_start, p_t), ...] -> (C array or None, count)."""
+    if not prefills:
+        return None, 0
+    arr = (mx_prefill * len(prefills))(*[mx_prefill(int(a), int(b), int(c)) for a, b, c in prefills])
+    return arr, len(prefills)
 
 
 class mx_layer_bufs(ctypes.Structure):
@@ -93,8 +106,8 @@ def load():
 
 def plan_work(*, num_q_heads, num_kv_heads=8, num_pages, num_seqs, max_pages_per_seq,
               max_tokens, max_decodes, decode_seq_ids, decode_ctx_lens, prefill_seq_id=-1,
-              chunk_start=0, p_t=0, num_sms=152, split_keys=0, piece_tiles=0, pdl=1,
-              max_items=1 << 16):
+              chunk_start=0, p_t=0, prefills=None, num_sms=152, split_keys=0, piece_tiles=0,
+              pdl=1, max_items=1 << 16):
     """The work list a launch would run (host only, no device): items
     int32 [n, 4] in claim order, decodes int32 [n_decodes, 4] and the counts
     (n_items, prefill items, split_keys, piece_tiles)."""
@@ -103,8 +116,10 @@ def plan_work(*, num_q_heads, num_kv_heads=8, num_pages, num_seqs, max_pages_per
                    max_tokens, max_decodes)
     ids = np.ascontiguousarray(np.asarray(decode_seq_ids, dtype=np.int32))
     lens = np.ascontiguousarray(np.asarray(decode_ctx_lens, dtype=np.int32))
+    pf_arr, n_pf = _prefill_array(prefills)
     desc = mx_iter_desc(ids.ctypes.data if len(ids) else None, lens.ctypes.data if len(lens) else None,
-                        len(lens), int(prefill_seq_id), int(chunk_start), int(p_t), None, None)
+                        len(lens), int(prefill_seq_id), int(chunk_start), int(p_t), None, None,
+                        n_pf, ctypes.cast(pf_arr, ctypes.c_void_p) if pf_arr is not None else None)
     items = np.zeros((max(max_items, 1), 4), np.int32)
     decs = np.zeros((max(len(lens), 1), 4), np.int32)
     counts = np.zeros(4, np.int32)
@@ -186,16 +201,19 @@ class Context:
                                            _ptr(k_pool), _ptr(v_pool), _stream_handle(stream)))
 
     def make_desc(self, *, decode_seq_ids, decode_ctx_lens, prefill_seq_id=-1,
-                  chunk_start=0, p_t=0, page_table, slots):
-        """Descriptor with HOST decode arrays and DEVICE page_table/slots.
-        The returned object keeps the host arrays alive."""
+                  chunk_start=0, p_t=0, page_table, slots, prefills=None):
+        """Descriptor with HOST decode arrays and DEVICE page_table/slots;
+        several prefill chunks as ``prefills`` = [(seq, chunk_start, p_t),
+        ...].  The returned object keeps the host arrays alive."""
         ids = np.ascontiguousarray(np.asarray(decode_seq_ids, dtype=np.int32))
         lens = np.ascontiguousarray(np.asarray(decode_ctx_lens, dtype=np.int32))
+        pf_arr, n_pf = _prefill_array(prefills)
         d = mx_iter_desc(ids.ctypes.data if len(ids) else None,
                          lens.ctypes.data if len(lens) else None, len(lens),
                          int(prefill_seq_id), int(chunk_start), int(p_t),
-                         _ptr(page_table), _ptr(slots))
-        d._keep = (ids, lens)
+                         _ptr(page_table), _ptr(slots), n_pf,
+                         ctypes.cast(pf_arr, ctypes.c_void_p) if pf_arr is not None else None)
+        d._keep = (ids, lens, pf_arr)
         return d
 
     @staticmethod

@@ -117,6 +117,8 @@ int cuda_fail(mx_ctx *c, cudaError_t e, const char *what)
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct Plan {
+    const PrefillInfo *pre_dev = nullptr;
+    int n_prefills = 0;
     int n_items = 0;
     int n_prefill = 0;
     int split_keys = 0;
@@ -129,7 +131,8 @@ struct Plan {
 // (both 16-byte records), uploaded with one copy.
 size_t plan_capacity_bytes(const mx_ctx *c)
 {
-    return (size_t)std::max(c->g.max_decodes, 1) * sizeof(DecodeInfo) + (size_t)c->max_items * sizeof(int4);
+    return (size_t)std::max(c->g.max_decodes, 1) * sizeof(DecodeInfo) + (size_t)kMaxPrefills * sizeof(PrefillInfo) +
+           (size_t)c->max_items * sizeof(int4);
 }
 
 // The geometries the kernels support.
@@ -170,10 +173,30 @@ int validate_desc(const mx_geom &g, const mx_iter_desc *d, bool need_tables, std
         return fail_to(err, MX_EINVAL, "negative n_decodes, p_t or chunk_start");
     if (d->n_decodes > g.max_decodes)
         return fail_to(err, MX_ECAPACITY, "n_decodes %d > max_decodes %d", d->n_decodes, g.max_decodes);
-    if ((int64_t)d->n_decodes + d->p_t > g.max_tokens)
-        return fail_to(err, MX_ECAPACITY, "n_decodes + p_t = %lld > max_tokens %d",
-                       (long long)d->n_decodes + d->p_t, g.max_tokens);
+    if (d->n_prefills < 0 || d->n_prefills > kMaxPrefills || (d->n_prefills > 0 && !d->prefills))
+        return fail_to(err, MX_EINVAL, "n_prefills %d outside [0, %d] or prefills null", d->n_prefills,
+                       kMaxPrefills);
+    if (d->n_prefills > 0 && (d->p_t != 0 || d->chunk_start != 0))
+        return fail_to(err, MX_EINVAL, "with n_prefills > 0, p_t and chunk_start must be 0");
     const int64_t cap = (int64_t)g.max_pages_per_seq * kPage;
+    int64_t n_tok = d->n_decodes + (int64_t)d->p_t;
+    for (int f = 0; f < d->n_prefills; ++f) {
+        const mx_prefill &x = d->prefills[f];
+        if (x.p_t <= 0 || x.chunk_start < 0)
+            return fail_to(err, MX_EINVAL, "prefill %d: p_t %d <= 0 or chunk_start %d < 0", f, x.p_t,
+                           x.chunk_start);
+        if (x.seq_id < 0 || x.seq_id >= g.num_seqs)
+            return fail_to(err, MX_EINVAL, "prefill %d: seq id %d outside [0, %d)", f, x.seq_id, g.num_seqs);
+        if ((int64_t)x.chunk_start + x.p_t > cap)
+            return fail_to(err, MX_ECAPACITY, "prefill %d: chunk end %lld exceeds %lld page-table slots", f,
+                           (long long)x.chunk_start + x.p_t, (long long)cap);
+        for (int e = 0; e < f; ++e)
+            if (d->prefills[e].seq_id == x.seq_id)
+                return fail_to(err, MX_EINVAL, "prefills %d and %d are chunks of the same sequence", e, f);
+        n_tok += x.p_t;
+    }
+    if (n_tok > g.max_tokens)
+        return fail_to(err, MX_ECAPACITY, "n_tokens = %lld > max_tokens %d", (long long)n_tok, g.max_tokens);
     if (d->n_decodes > 0 && (!d->decode_seq_ids || !d->decode_ctx_lens))
         return fail_to(err, MX_EINVAL, "decode_seq_ids / decode_ctx_lens are null");
     for (int i = 0; i < d->n_decodes; ++i) {
@@ -192,9 +215,43 @@ int validate_desc(const mx_geom &g, const mx_iter_desc *d, bool need_tables, std
             return fail_to(err, MX_ECAPACITY, "chunk end %lld exceeds %lld page-table slots",
                            (long long)d->chunk_start + d->p_t, (long long)cap);
     }
-    if (need_tables && d->n_decodes + d->p_t > 0 && (!d->page_table || !d->slots))
+    if (need_tables && n_tok > 0 && (!d->page_table || !d->slots))
         return fail_to(err, MX_EINVAL, "page_table / slots are null");
     return MX_OK;
+}
+
+// The iteration's prefill chunks in token order (the single chunk of the
+// descriptor, or its array), with their token and query-tile offsets.
+std::vector<PrefillInfo> prefill_list(const mx_iter_desc *d)
+{
+    std::vector<PrefillInfo> v;
+    int tb = d->n_decodes, tile = 0;
+    auto add = [&](int seq, int cs, int p) {
+        PrefillInfo x{};
+        x.seq = seq;
+        x.chunk_start = cs;
+        x.p_t = p;
+        x.token_base = tb;
+        x.tile_base = tile;
+        v.push_back(x);
+        tb += p;
+        tile += (p + kTileM - 1) / kTileM;
+    };
+    if (d->n_prefills > 0) {
+        for (int f = 0; f < d->n_prefills; ++f)
+            add(d->prefills[f].seq_id, d->prefills[f].chunk_start, d->prefills[f].p_t);
+    } else if (d->p_t > 0) {
+        add(d->prefill_seq_id, d->chunk_start, d->p_t);
+    }
+    return v;
+}
+
+int64_t token_count(const mx_iter_desc *d)
+{
+    int64_t n = d->n_decodes + (int64_t)d->p_t;
+    for (int f = 0; f < d->n_prefills; ++f)
+        n += d->prefills[f].p_t;
+    return n;
 }
 
 int validate(mx_ctx *c, const mx_iter_desc *d)
@@ -229,16 +286,21 @@ struct PlanKnobs {
     int max_items;         // capacity of the items array
 };
 struct WorkList {
-    int n_items = 0, n_prefill = 0, split_keys = 0, piece_tiles = 0;
+    int n_items = 0, n_prefill = 0, n_prefills = 0, split_keys = 0, piece_tiles = 0;
 };
 
 // a1: the per-iteration work list, on the host, into dec[n_decodes] and
 // items[].  Prefill tiles first, heaviest (latest rows, most keys) first;
 // then decode splits, longest first.
 int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k, DecodeInfo *dec,
-                    int4 *items, WorkList *out, std::string *err)
+                    PrefillInfo *pre, int4 *items, WorkList *out, std::string *err)
 {
     const int hkv = g.num_kv_heads, hq = g.num_q_heads;
+    const std::vector<PrefillInfo> pfs = prefill_list(d);
+    const int n_pf = (int)pfs.size();
+    int n_qt = 0;  // query tiles over all chunks
+    for (const PrefillInfo &x : pfs)
+        n_qt += (x.p_t + kTileM - 1) / kTileM;
     const int nd = d->n_decodes;
     int64_t total_keys = 0;
     for (int i = 0; i < nd; ++i)
@@ -256,8 +318,7 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
         // the optimum there).  With independent layers (MX_OPT_PDL = 2) the
         // next layer fills the tail, so the splits stay long.
         double per_sm = 1.5;
-        if (d->p_t > 0) {
-            const int n_qt = (d->p_t + kTileM - 1) / kTileM;
+        if (n_qt > 0) {
             static const double kBeside[3] = {3.5, 3.0, 2.0};
             per_sm = k.pdl == 2 ? 1.0 : (n_qt <= 3 ? kBeside[n_qt - 1] : 1.0);
         }
@@ -284,11 +345,12 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
     // Prefill tiles, split along their key tiles into pieces of at most
     // piece_tiles tiles so that long causal rows spread over several SMs.
     int n = 0;
-    const int n_qt = (d->p_t + kTileM - 1) / kTileM;
-    const int nA = (d->chunk_start + kTileN - 1) / kTileN;
     int64_t pre_work = 0;
-    for (int t = 0; t < n_qt; ++t)
-        pre_work += (int64_t)(nA + t + 1) * hq;
+    for (const PrefillInfo &x : pfs) {
+        const int nA = (x.chunk_start + kTileN - 1) / kTileN;
+        for (int t = 0; t < (x.p_t + kTileM - 1) / kTileM; ++t)
+            pre_work += (int64_t)(nA + t + 1) * hq;
+    }
     // Splitting costs a partial write and a merge; it pays only when the
     // chunk has too few tiles to occupy the GPU (short chunks deep into a
     // long prompt), so tiles are split only then, into >= 48-tile pieces.
@@ -301,10 +363,13 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
     }
     auto count_pre_parts = [&](int pc) {
         int64_t parts = 0;
-        for (int t = 0; t < n_qt; ++t) {
-            const int ns = (nA + t + 1 + pc - 1) / pc;
-            if (ns > 1)
-                parts += (int64_t)ns * hq;
+        for (const PrefillInfo &x : pfs) {
+            const int nA = (x.chunk_start + kTileN - 1) / kTileN;
+            for (int t = 0; t < (x.p_t + kTileM - 1) / kTileM; ++t) {
+                const int ns = (nA + t + 1 + pc - 1) / pc;
+                if (ns > 1)
+                    parts += (int64_t)ns * hq;
+            }
         }
         return parts;
     };
@@ -314,16 +379,20 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
     std::vector<PItem> pitems;
     pitems.reserve(64);
     int pre_part = 0;
-    for (int t = n_qt - 1; t >= 0; --t) {
-        const int nT = nA + t + 1;
-        const int ns = (nT + piece - 1) / piece;
-        for (int h = 0; h < hq; ++h) {
-            const int base = ns > 1 ? pre_part : 0;
-            if (ns > 1)
-                pre_part += ns;
-            for (int s2 = 0; s2 < ns; ++s2) {
-                const int len = (int)((int64_t)(s2 + 1) * nT / ns - (int64_t)s2 * nT / ns);
-                pitems.push_back({len, prefill_item_code(t, h, s2, ns, base)});
+    for (int f = 0; f < n_pf; ++f) {
+        pre[f] = pfs[f];
+        const int nA = (pfs[f].chunk_start + kTileN - 1) / kTileN;
+        for (int t = (pfs[f].p_t + kTileM - 1) / kTileM - 1; t >= 0; --t) {
+            const int nT = nA + t + 1;
+            const int ns = (nT + piece - 1) / piece;
+            for (int h = 0; h < hq; ++h) {
+                const int base = ns > 1 ? pre_part : 0;
+                if (ns > 1)
+                    pre_part += ns;
+                for (int s2 = 0; s2 < ns; ++s2) {
+                    const int len = (int)((int64_t)(s2 + 1) * nT / ns - (int64_t)s2 * nT / ns);
+                    pitems.push_back({len, prefill_item_code(f, t, h, s2, ns, base)});
+                }
             }
         }
     }
@@ -368,6 +437,7 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
 
     out->n_items = n;
     out->n_prefill = n_prefill;
+    out->n_prefills = n_pf;
     out->split_keys = split;
     out->piece_tiles = piece;
     return MX_OK;
@@ -386,11 +456,13 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     }
     uint8_t *host = c->plan_host[slot];
     DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(host);
-    const size_t items_off = (size_t)d->n_decodes * sizeof(DecodeInfo);
+    const size_t pre_off = (size_t)d->n_decodes * sizeof(DecodeInfo);
+    PrefillInfo *pre = reinterpret_cast<PrefillInfo *>(host + pre_off);
+    const size_t items_off = pre_off + (size_t)kMaxPrefills * sizeof(PrefillInfo);
     int4 *items = reinterpret_cast<int4 *>(host + items_off);
     const PlanKnobs knobs{c->num_sms, c->split_keys_opt, c->piece_tiles_opt, c->pdl, c->max_items};
     WorkList wl;
-    int rc = build_work_list(c->g, d, knobs, dec, items, &wl, &c->last_error);
+    int rc = build_work_list(c->g, d, knobs, dec, pre, items, &wl, &c->last_error);
     if (rc)
         return rc;
     const int n = wl.n_items;
@@ -420,6 +492,8 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     out->slot = slot;
     out->items_dev = reinterpret_cast<const int4 *>(c->plan_dev[slot] + items_off);
     out->dec_dev = reinterpret_cast<const DecodeInfo *>(c->plan_dev[slot]);
+    out->pre_dev = reinterpret_cast<const PrefillInfo *>(c->plan_dev[slot] + pre_off);
+    out->n_prefills = wl.n_prefills;
     c->last_items = n;
     c->last_split = wl.split_keys;
     c->last_prefill_items = wl.n_prefill;
@@ -445,7 +519,7 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
 {
     const mx_geom &g = c->g;
     std::memset(P, 0, sizeof *P);
-    const int n_tok = d->n_decodes + d->p_t;
+    const int n_tok = (int)token_count(d);
     P->q = static_cast<const uint16_t *>(b->q);
     P->k = static_cast<const uint16_t *>(b->k);
     P->v = static_cast<const uint16_t *>(b->v);
@@ -467,9 +541,8 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->err = c->err;
     P->n_items = pl.n_items;
     P->n_decodes = d->n_decodes;
-    P->prefill_seq = d->p_t > 0 ? d->prefill_seq_id : 0;
-    P->chunk_start = d->chunk_start;
-    P->p_t = d->p_t;
+    P->pre = pl.pre_dev;
+    P->n_prefills = pl.n_prefills;
     P->hq = g.num_q_heads;
     P->hkv = g.num_kv_heads;
     P->n_rep = g.num_q_heads / g.num_kv_heads;
@@ -598,7 +671,8 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     c->g = *g;
     c->device = device;
     c->num_sms = prop.multiProcessorCount;
-    const int max_qtiles = std::max((g->max_tokens + kTileM - 1) / kTileM, 1);
+    // every chunk may end in a ragged tile
+    const int max_qtiles = std::max((g->max_tokens + kTileM - 1) / kTileM, 1) + kMaxPrefills - 1;
     const int max_prefill_items = max_qtiles * g->num_q_heads + kPrePartSlots;
     c->max_items = max_prefill_items + kPartSlots + std::max(g->max_decodes, 1) * g->num_kv_heads;
 
@@ -741,7 +815,7 @@ int mx_mixed_attention(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b,
     int rc = validate(c, d);
     if (rc)
         return rc;
-    const int n_tok = d->n_decodes + d->p_t;
+    const int n_tok = (int)token_count(d);
     if ((rc = validate_bufs(c, b, n_tok)))
         return rc;
     if (n_tok == 0)
@@ -771,7 +845,7 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     if (n_layers < 0 || (n_layers > 0 && !layers))
         return fail(c, MX_EINVAL, "bad n_layers / layers");
     const bool timed = device_us_out != nullptr;
-    const int n_tok = d->n_decodes + d->p_t;
+    const int n_tok = (int)token_count(d);
     for (int l = 0; l < n_layers; ++l)
         if ((rc = validate_bufs(c, layers + l, n_tok)))
             return rc;
@@ -899,10 +973,11 @@ int mx_plan_work(const mx_geom *geom, const mx_iter_desc *desc, int32_t num_sms,
         rc = fail_to(&err, MX_EINVAL, "decodes is null");
     if (rc == MX_OK) {
         std::vector<DecodeInfo> dec((size_t)std::max(desc->n_decodes, 1));
+        std::vector<PrefillInfo> pre(kMaxPrefills);
         std::vector<int4> it((size_t)std::max(max_items, 1));
         const PlanKnobs knobs{num_sms, split_keys_opt, piece_tiles_opt, pdl, max_items};
         WorkList wl;
-        rc = build_work_list(*geom, desc, knobs, dec.data(), it.data(), &wl, &err);
+        rc = build_work_list(*geom, desc, knobs, dec.data(), pre.data(), it.data(), &wl, &err);
         if (rc == MX_OK) {
             if (wl.n_items > 0)
                 std::memcpy(items, it.data(), (size_t)wl.n_items * sizeof(int4));

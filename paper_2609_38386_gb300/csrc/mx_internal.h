@@ -50,19 +50,31 @@ constexpr uint32_t kTmemO = kSBuf * 128;
 
 enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
 
+// Prefill chunks of one iteration (several prompts' chunks may share it).
+constexpr int kMaxPrefills = 16;
+struct PrefillInfo {
+    int32_t seq;          // page-table row
+    int32_t chunk_start;  // position of the chunk's row 0
+    int32_t p_t;          // chunk rows
+    int32_t token_base;   // token index of row 0 in q/k/v/out/slots
+    int32_t tile_base;    // its first query tile, counted over all chunks
+    int32_t pad[3];
+};
+
 // Work-item encodings (int4):
-//   prefill: {ITEM_PREFILL, t | hq << 16, s | n_s << 16, partial slot base}
-//            piece s of n_s of query tile t (rows [128t, 128t+128)) of head hq;
-//            the tile's key tiles are split evenly between its n_s pieces.
+//   prefill: {ITEM_PREFILL | chunk f << 4, t | hq << 16, s | n_s << 16,
+//             partial slot base}: piece s of n_s of query tile t (rows
+//            [128t, 128t+128) of chunk f) of head hq; the tile's key tiles are
+//            split evenly between its n_s pieces.
 //   decode:  {ITEM_DECODE | kv head << 4 | split index << 11 | split
 //             length / 16 << 23, decode index, page-table row, cached tokens}:
 //             split s of decode i covers keys [s * len, (s + 1) * len) of
 //             [0, ctx]; the row, length and split size travel in the item so
 //             that the page-id loads need no other lookup first
-__host__ __device__ inline int4 prefill_item_code(int t, int hq, int s, int n_s, int part_base)
+__host__ __device__ inline int4 prefill_item_code(int f, int t, int hq, int s, int n_s, int part_base)
 {
     int4 r;
-    r.x = ITEM_PREFILL;
+    r.x = ITEM_PREFILL | (f << 4);
     r.y = t | (hq << 16);
     r.z = s | (n_s << 16);
     r.w = part_base;
@@ -118,9 +130,8 @@ struct LayerParams {
 
     int32_t n_items;
     int32_t n_decodes;
-    int32_t prefill_seq;
-    int32_t chunk_start;
-    int32_t p_t;
+    const PrefillInfo *pre; // [n_prefills] prefill chunks
+    int32_t n_prefills;
     int32_t hq, hkv, n_rep;
     int32_t num_pages, max_pages;
     int32_t split_keys;    // keys per decode split (multiple of 128)

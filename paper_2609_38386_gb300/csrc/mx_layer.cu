@@ -43,6 +43,7 @@ struct Misc {
     int32_t item_idx[2];
     int32_t abort;
     int32_t last;
+    PrefillInfo pre[kMaxPrefills];  // the launch's prefill chunks
 };
 static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
 static_assert(kVStages == 2, "V stage c % 2 is released by the odone barrier c & 1");
@@ -269,8 +270,17 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
         l0 += p0 + p2;
         l1 += p1 + p3;
         // P^T as the B operand (keys x query rows): transpose the 8x8 blocks
-        const uint32_t b0 = movmatrix_t(pack_bf16(p0, p1));
-        const uint32_t b1 = movmatrix_t(pack_bf16(p2, p3));
+        const uint32_t h01 = pack_bf16(p0, p1), h23 = pack_bf16(p2, p3);
+        const uint32_t b0 = movmatrix_t(h01);
+        const uint32_t b1 = movmatrix_t(h23);
+        // A decode of at most 16 keys takes P as hi + lo (p minus its bf16
+        // rounding): with so few keys one weight's rounding shows in O.
+        const bool lo = n < kPage;
+        uint32_t c0 = 0u, c1 = 0u;
+        if (lo) {
+            c0 = movmatrix_t(pack_bf16(p0 - bf16lo(h01), p1 - bf16hi(h01)));
+            c1 = movmatrix_t(pack_bf16(p2 - bf16lo(h23), p3 - bf16hi(h23)));
+        }
         // O^T (128 d x 8 rows) += V^T (128 x 16 keys) * P^T (16 x 8)
         {
             const int mi = lane >> 3;
@@ -281,6 +291,7 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
                 uint32_t a0, a1, a2, a3;
                 ldsm_x4_t(vbase + key * 256 + ((chunk ^ (key & 7)) << 4), a0, a1, a2, a3);
                 mma_bf16_16816(acc[mt], a0, a1, a2, a3, b0, b1);
+
             }
         }
         __syncwarp();
@@ -411,7 +422,12 @@ __device__ __forceinline__ float row_max(const uint32_t (&sv)[128])
 
 // p = 2^(s*scale - m) of one S row as bf16 pairs into TMEM at taddr (64
 // columns), and the row sum of p in 4 packed pair chains.
-__device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float sl, float nm, uint32_t taddr)
+// With lo set, the low-order part of P (p minus its bf16 rounding) goes to
+// the second half of S_c as well: rows with only a few keys (the first rows
+// of a prompt) would show the rounding of a single weight of P in the
+// output, so their P.V takes P as hi + lo.
+__device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float sl, float nm, uint32_t taddr,
+                                               bool lo)
 {
     float rs8[8];
 #pragma unroll
@@ -430,8 +446,95 @@ __device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float 
             pk[cc] = pack_bf16(e0, e1);
         }
         tmem_st32(taddr + 32 * half, pk);
+        if (lo) {
+#pragma unroll
+            for (int cc = 0; cc < 32; ++cc) {
+                const int k0 = 64 * half + 2 * cc;
+                float x0, x1;
+                ffma2(x0, x1, __uint_as_float(sv[k0]), __uint_as_float(sv[k0 + 1]), sl, sl, nm, nm);
+                const float e0 = ex2(x0), e1 = ex2(x1);
+                pk[cc] = pack_bf16(e0 - bf16lo(pk[cc]), e1 - bf16hi(pk[cc]));
+            }
+            tmem_st32(taddr + 64 + 32 * half, pk);
+        }
     }
     return ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
+}
+
+// 16-byte chunk c (8 elements) of row `row` of a 128 x 128 bf16 tile held as
+// two SW128 halves of 64 columns (128-byte rows), as the TMA loads write it.
+__device__ __forceinline__ uint4 sw128_chunk(uint32_t base, int row, int c)
+{
+    const uint32_t a = base + (uint32_t)(c >> 3) * kHalfTile + row * 128 + ((((c & 7) ^ (row & 7))) << 4);
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+
+// Chunk row r < 16 of a chunk that starts at position 0 attends only keys
+// 0..r.  With so few keys the bf16 rounding of a single weight of P would
+// show in the output, so such a row is recomputed here in fp32 from the Q,
+// K and V tiles still in shared memory (the item's only key tile) and its
+// output row overwritten.
+__device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKt, uint32_t sVt, int r, float sl,
+                                                uint16_t *orow)
+{
+    float s[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+        s[k] = 0.f;
+#pragma unroll 1
+    for (int c = 0; c < 16; ++c) {
+        const uint4 q4 = sw128_chunk(sQ, r, c);
+        const uint32_t qw[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            if (k <= r) {
+                const uint4 k4 = sw128_chunk(sKt, k, c);
+                const uint32_t kw[4] = {k4.x, k4.y, k4.z, k4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    s[k] += bf16lo(qw[e]) * bf16lo(kw[e]) + bf16hi(qw[e]) * bf16hi(kw[e]);
+            }
+        }
+    }
+    float m = neg_inf();
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+        if (k <= r)
+            m = fmaxf(m, s[k] * sl);
+    float l = 0.f;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        s[k] = k <= r ? ex2(s[k] * sl - m) : 0.f;
+        l += s[k];
+    }
+    const float inv = 1.0f / l;
+#pragma unroll 1
+    for (int c = 0; c < 16; ++c) {
+        float acc[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            acc[e] = 0.f;
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            if (k <= r) {
+                const uint4 v4 = sw128_chunk(sVt, k, c);
+                const uint32_t vw[4] = {v4.x, v4.y, v4.z, v4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    acc[2 * e] += s[k] * bf16lo(vw[e]);
+                    acc[2 * e + 1] += s[k] * bf16hi(vw[e]);
+                }
+            }
+        }
+        uint4 o4;
+        o4.x = pack_bf16(acc[0] * inv, acc[1] * inv);
+        o4.y = pack_bf16(acc[2] * inv, acc[3] * inv);
+        o4.z = pack_bf16(acc[4] * inv, acc[5] * inv);
+        o4.w = pack_bf16(acc[6] * inv, acc[7] * inv);
+        reinterpret_cast<uint4 *>(orow)[c] = o4;
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -440,12 +543,13 @@ __device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float 
 // the chunk's own keys read from the k/v inputs.
 // ---------------------------------------------------------------------------
 __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem,
-                             int t, int hq, int kt0, int kt1, int part_slot, uint32_t tile0,
-                             uint32_t item_no)
+                             const PrefillInfo &pf, int t, int hq, int kt0, int kt1, int part_slot,
+                             uint32_t tile0, uint32_t item_no)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int kvh = hq / P.n_rep;
-    const int cs = P.chunk_start, p = P.p_t, nd = P.n_decodes;
+    // tb: token index of the chunk's row 0 in q/k/v/out/slots
+    const int cs = pf.chunk_start, p = pf.p_t, tb = pf.token_base;
     const int nA = (cs + kTileN - 1) / kTileN;
     const int nT = kt1 - kt0;  // key tiles of this piece: global tiles kt0 + i
     const uint32_t sbase = smem_u32(smem);
@@ -462,8 +566,8 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         if (isK && lane == 0) {
             fence_proxy_async_smem();
             mbar_expect_tx(bar_q, kTileBytes);
-            tma_load_3d(sQ, &P.tm_q, bar_q, 0, hq, nd + kTileM * t);
-            tma_load_3d(sQ + kHalfTile, &P.tm_q, bar_q, 64, hq, nd + kTileM * t);
+            tma_load_3d(sQ, &P.tm_q, bar_q, 0, hq, tb + kTileM * t);
+            tma_load_3d(sQ + kHalfTile, &P.tm_q, bar_q, 64, hq, tb + kTileM * t);
         }
         const int nst = isK ? kKStages : kVStages;
         const uint32_t ring = isK ? sK : sV;
@@ -478,7 +582,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         // Page ids of cached tiles, four tiles (32 pages, one per lane) per
         // load, fetched one batch ahead: a page-table read under load takes
         // about as long as a whole tile, so it must not sit in the issue loop.
-        const int32_t *prow = P.page_table + (size_t)P.prefill_seq * P.max_pages;
+        const int32_t *prow = P.page_table + (size_t)pf.seq * P.max_pages;
         auto fetch_pids = [&](int i0) {
             const int lp = (kt0 + i0 + (lane >> 3)) * 8 + (lane & 7);
             int pid = -1;
@@ -530,7 +634,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                             tma_load_2d(dst + hf * kHalfTile + pg * 2048, tm_pool, fb, hf * 64, y);
                     }
                 } else {
-                    const int z = nd + kTileN * (gi - nA);
+                    const int z = tb + kTileN * (gi - nA);
 #pragma unroll
                     for (int hf = 0; hf < 2; ++hf)
                         tma_load_3d(dst + hf * kHalfTile, tm_in, fb, hf * 64, kvh, z);
@@ -587,6 +691,12 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                     for (int kk = 0; kk < 8; ++kk)  // 16 keys of MN-major V: +2 KiB
                         tc_mma_ts(tmem + kTmemO, pa + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4), kIdescO,
                                   (j > 0 || kk > 0) ? 1u : 0u);
+                    if (false) {  // the low-order part of P
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk)
+                            tc_mma_ts(tmem + kTmemO, pa + 64 + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4),
+                                      kIdescO, 1u);
+                    }
                     tc_commit(smem_u32(&misc->bar_odone[c & 1]));  // also frees V stage st
                 }
             }
@@ -612,10 +722,10 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             const int u = r / P.n_rep, sub = r % P.n_rep;
             const int ja = kTileM * t + (hq % P.n_rep) * per + u;   // chunk row of this thread's token
             const bool app = kt0 == 0 && ja < p;
-            const size_t arow = ((size_t)(nd + ja) * P.hkv + kvh) * kHeadDim;
+            const size_t arow = ((size_t)(tb + ja) * P.hkv + kvh) * kHeadDim;
             int slot = -1;
             if (app)
-                slot = __ldg(P.slots + nd + ja);
+                slot = __ldg(P.slots + tb + ja);
             for (int b = 0; app && b < npc; b += 16) {
                 uint4 av[16];
 #pragma unroll
@@ -672,7 +782,8 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
             // P_c (the A operand of P.V) goes over the first 64 columns of
             // S_c, whose buffer P_{c-3} held: S_c was issued after
             // P_{c-3} V_{c-3}, so its completion covers that read too.
-            const float rs = row_exp_store(sv, sl, nm, tl + sb * 128);
+            // rows with fewer than 17 keys (the first rows of a prompt) take P as hi + lo
+            const float rs = row_exp_store(sv, sl, nm, tl + sb * 128, false);
             // The O correction comes after P, when the scores are no longer
             // live, and before P_c is released to the MMA issuer.
             if (rescale && i > 0) {
@@ -737,7 +848,7 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
         } else {
             tc_fence_after();
             const float inv = 1.0f / l_run;
-            uint16_t *orow = P.out + ((size_t)(nd + j) * P.hq + hq) * kHeadDim;
+            uint16_t *orow = P.out + ((size_t)(tb + j) * P.hq + hq) * kHeadDim;
 #pragma unroll
             for (int gq = 0; gq < 4; ++gq) {
                 uint32_t o[32];
@@ -755,18 +866,28 @@ __device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, ui
                     }
                 }
             }
+            // the first 16 rows of a prompt: exact fp32 recomputation (the
+            // item has one key tile, tile0's K and V stages hold it)
+            if (cs == 0 && t == 0 && r < kPage && j < p) {
+                // the tiles' TMA writes, observed on their own (completed) barriers
+                if (mbar_wait(bar_q, item_no & 1, abort, tmo) &&
+                    mbar_wait(smem_u32(&misc->bar_kfull[tile0 % kKStages]), (tile0 / kKStages) & 1, abort, tmo) &&
+                    mbar_wait(smem_u32(&misc->bar_pfull[tile0 % kSBuf]), (tile0 / kSBuf) & 1, abort, tmo))
+                    short_row_exact(sQ, sK + (tile0 % kKStages) * kTileBytes, sV + (tile0 % kVStages) * kTileBytes,
+                                    r, sl, orow);
+            }
         }
     }
 }
 
 // Merge the n_s pieces of prefill tile (t, hq) if this CTA's piece arrived
 // last (no waiting): out = sum_s w_s O_s / sum_s w_s, w_s = 2^(lse_s - max).
-__device__ void prefill_merge(const LayerParams &P, Misc *misc, int t, int hq, int n_s,
-                              int part_base)
+__device__ void prefill_merge(const LayerParams &P, Misc *misc, const PrefillInfo &pf, int t, int hq,
+                              int n_s, int part_base)
 {
     const int tid = threadIdx.x;
     if (tid == 0) {
-        const uint32_t prev = atomicAdd(P.pre_cnt + t * P.hq + hq, 1u);
+        const uint32_t prev = atomicAdd(P.pre_cnt + (pf.tile_base + t) * P.hq + hq, 1u);
         misc->last = (prev == (uint32_t)(n_s - 1)) ? 1 : 0;
     }
     __syncthreads();
@@ -774,7 +895,7 @@ __device__ void prefill_merge(const LayerParams &P, Misc *misc, int t, int hq, i
         __threadfence();
         const int r = tid >> 1, half = tid & 1;
         const int j = kTileM * t + r;
-        if (j < P.p_t) {
+        if (j < pf.p_t) {
             float M = neg_inf();
             for (int s = 0; s < n_s; ++s)
                 M = fmaxf(M, __ldcg(P.pre_lse + (size_t)(part_base + s) * kTileM + r));
@@ -802,7 +923,7 @@ __device__ void prefill_merge(const LayerParams &P, Misc *misc, int t, int hq, i
                     }
                 }
                 uint4 *dst = reinterpret_cast<uint4 *>(
-                    P.out + ((size_t)(P.n_decodes + j) * P.hq + hq) * kHeadDim + d0);
+                    P.out + ((size_t)(pf.token_base + j) * P.hq + hq) * kHeadDim + d0);
 #pragma unroll
                 for (int x = 0; x < 4; ++x)
                     dst[x] = make_uint4(pack_bf16(acc[8 * x] * inv, acc[8 * x + 1] * inv),
@@ -852,6 +973,8 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         tmem_alloc(smem_u32(&misc->tmem_base), kTmemCols);
         tmem_relinquish();
     }
+    if (tid >= 64 && tid < 64 + P.n_prefills)
+        misc->pre[tid - 64] = P.pre[tid - 64];
     // Consecutive launches use alternate workspace sets, and the launch two
     // back has completed before this one was launched (see the end of the
     // kernel), so work starts at once, beside the previous layer's tail.
@@ -885,13 +1008,15 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         if (tid == 0)
             misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
         const int4 it = P.items[idx];
-        int merge_t = -1, merge_hq = 0, merge_ns = 1;
-        if (it.x == ITEM_PREFILL) {
+        int merge_t = -1, merge_hq = 0, merge_ns = 1, merge_f = 0;
+        if ((it.x & 0xF) == ITEM_PREFILL) {
+            const int f = (int)((uint32_t)it.x >> 4);
+            const PrefillInfo &pf = misc->pre[f];
             const int t = it.y & 0xFFFF, hq = it.y >> 16;
             const int s = it.z & 0xFFFF, ns = it.z >> 16;
-            const int nT = (P.chunk_start + kTileN - 1) / kTileN + t + 1;
+            const int nT = (pf.chunk_start + kTileN - 1) / kTileN + t + 1;
             const int kt0 = (int)((long long)s * nT / ns), kt1 = (int)((long long)(s + 1) * nT / ns);
-            prefill_item(P, smem, misc, tmem, t, hq, kt0, kt1, ns > 1 ? it.w + s : -1, tile_cnt,
+            prefill_item(P, smem, misc, tmem, pf, t, hq, kt0, kt1, ns > 1 ? it.w + s : -1, tile_cnt,
                          item_no);
             tile_cnt += kt1 - kt0;
             item_no += 1;
@@ -899,6 +1024,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
                 merge_t = t;
                 merge_hq = hq;
                 merge_ns = ns;
+                merge_f = f;
             }
         } else {
             const uint32_t dx = (uint32_t)it.x;
@@ -910,7 +1036,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         __syncthreads();
         tc_fence_after();
         if (merge_t >= 0 && !misc->abort)
-            prefill_merge(P, misc, merge_t, merge_hq, merge_ns, it.w);
+            prefill_merge(P, misc, misc->pre[merge_f], merge_t, merge_hq, merge_ns, it.w);
         buf ^= 1;
     }
 

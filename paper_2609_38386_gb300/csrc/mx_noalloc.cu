@@ -55,7 +55,8 @@ constexpr size_t kOffWork = kOffMerge + kMergeBytes;  // [0] next item, [1] CTAs
 constexpr size_t kWorkBytes = 256;
 constexpr size_t kOffPlan = kOffWork + kWorkBytes;    // DecodeInfo[256], then int4 items[4096]
 constexpr size_t kPlanBytes = (size_t)kNaMaxDecodes * sizeof(DecodeInfo) + (size_t)kNaMaxItems * sizeof(int4);
-constexpr size_t kScratchBytes = kOffPlan + kPlanBytes;
+constexpr size_t kOffPre = kOffPlan + kPlanBytes;    // PrefillInfo of the one chunk
+constexpr size_t kScratchBytes = kOffPre + 256;
 
 }  // namespace
 
@@ -156,6 +157,9 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     const int nd = d->n_decodes, p = d->p_t;
     if (nd < 0 || p < 0 || d->chunk_start < 0)
         return report(err_buf, err_len, MX_EINVAL, "negative n_decodes, p_t or chunk_start");
+    if (d->n_prefills != 0)
+        return report(err_buf, err_len, MX_EINVAL,
+                      "several prefill chunks (n_prefills > 0) need a context: use mx_mixed_attention");
     if (nd > kNaMaxDecodes)
         return report(err_buf, err_len, MX_ECAPACITY, "n_decodes %d > %d (scratch limit)", nd,
                       kNaMaxDecodes);
@@ -222,7 +226,7 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     int n = 0;
     for (int t = n_qt - 1; t >= 0; --t)
         for (int h = 0; h < hq; ++h)
-            items[n++] = prefill_item_code(t, h, 0, 1, 0);
+            items[n++] = prefill_item_code(0, t, h, 0, 1, 0);
     const int n_prefill = n;
     int part = 0;
     for (int i = 0; i < nd; ++i) {
@@ -280,9 +284,14 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     P.err = P.work_cnt + 4;
     P.n_items = n;
     P.n_decodes = nd;
-    P.prefill_seq = p > 0 ? d->prefill_seq_id : 0;
-    P.chunk_start = d->chunk_start;
-    P.p_t = p;
+    PrefillInfo pre{};
+    pre.seq = d->prefill_seq_id;
+    pre.chunk_start = d->chunk_start;
+    pre.p_t = p;
+    pre.token_base = nd;
+    pre.tile_base = 0;
+    P.pre = reinterpret_cast<const PrefillInfo *>(sc + kOffPre);
+    P.n_prefills = p > 0 ? 1 : 0;
     P.hq = hq;
     P.hkv = hkv;
     P.n_rep = rep;
@@ -316,6 +325,8 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     cudaError_t e = cudaMemsetAsync(sc + kOffMerge, 0, kMergeBytes + kWorkBytes, s);
     if (e == cudaSuccess && nd > 0)
         e = cudaMemcpyAsync(sc + kOffPlan, dec, (size_t)nd * sizeof(DecodeInfo), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess && p > 0)
+        e = cudaMemcpyAsync(sc + kOffPre, &pre, sizeof pre, cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(const_cast<int4 *>(P.items), items, (size_t)n * sizeof(int4),
                             cudaMemcpyHostToDevice, s);

@@ -397,3 +397,82 @@ def test_bounded_wait_timeout_in_iteration(mode):
     fresh.close()
     for g, w in zip(got, want):
         np.testing.assert_array_equal(g, w)
+
+
+def _several_chunks_case(hq, ctxs, chunks, seed):
+    """Decodes plus several prompts' chunks (each its own sequence), seeded
+    host inputs: returns the layout, tokens, slots and initial pools."""
+    import synth
+    from synth import workload as wl
+    geom = wl.Geometry(hq)
+    nd = len(ctxs)
+    caps = [c + 1 for c in ctxs] + [cs + p for cs, p in chunks]
+    lay = wl.make_layout(geom, caps, seed=seed, spare_pages=1)
+    ps = geom.page_size
+    slots = [lay.page_table[i, c // ps] * ps + c % ps for i, c in enumerate(ctxs)]
+    for f, (cs, p) in enumerate(chunks):
+        slots += [lay.page_table[nd + f, (cs + j) // ps] * ps + (cs + j) % ps for j in range(p)]
+    n_tok = len(slots)
+    base = lambda s: synth.stream_base(seed, s)
+    q = synth.fill(base(1), (n_tok, hq, 128))
+    k = synth.fill(base(2), (n_tok, 8, 128))
+    v = synth.fill(base(3), (n_tok, 8, 128))
+    kp = synth.fill(base(4), lay.pool_shape())
+    vp = synth.fill(base(5), lay.pool_shape())
+    return geom, lay, np.asarray(slots, np.int32), q, k, v, kp, vp
+
+
+@pytest.mark.parametrize("hq,ctxs,chunks", [
+    (16, [300, 40], [(0, 100), (256, 200), (7000, 1)]),
+    (32, [], [(128, 128), (77, 300)]),
+    (64, [700, 3, 1500], [(1000, 300), (0, 640), (3000, 200), (10, 10)]),
+])
+def test_several_prefill_chunks(hq, ctxs, chunks):
+    """Several prompts' chunks in one launch (each a chunk of its own
+    sequence, rows after the decodes chunk by chunk), with ragged lengths,
+    a chunk at position 0 and a one-row chunk deep into its prompt (split
+    into key pieces): every row against the oracle, KV pages bit-exact."""
+    import oracle
+    from paper_2609_38386_gb300 import Context
+    geom, lay, slots, q, k, v, kp0, vp0 = _several_chunks_case(hq, ctxs, chunks, seed=hq + len(chunks))
+    nd = len(ctxs)
+    prefills = [(nd + f, cs, p) for f, (cs, p) in enumerate(chunks)]
+    ctx = Context(num_q_heads=hq, num_kv_heads=8, num_pages=lay.num_pages, num_seqs=lay.num_seqs,
+                  max_pages_per_seq=lay.max_pages, max_tokens=len(slots), max_decodes=max(nd, 1))
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda()
+    d_q, d_k, d_v, d_kp, d_vp = t(q), t(k), t(v), t(kp0), t(vp0)
+    d_out = torch.full((len(slots), hq, 128), 0x7FC1, dtype=torch.int16, device="cuda")
+    d_pt, d_sl = torch.from_numpy(lay.page_table).cuda(), torch.from_numpy(slots).cuda()
+    desc = ctx.make_desc(decode_seq_ids=list(range(nd)), decode_ctx_lens=ctxs, page_table=d_pt,
+                         slots=d_sl, prefills=prefills)
+    ctx.mixed_attention(desc, ctx.make_bufs(d_q, d_k, d_v, d_kp, d_vp, d_out))
+    ctx.sync_status()
+    torch.cuda.synchronize()
+    kp, vp = kp0.copy(), vp0.copy()
+    want, _ = oracle.mixed_attention(q=q, k=k, v=v, k_pool=kp, v_pool=vp, page_table=lay.page_table,
+                                     slots=slots, decode_seq_ids=np.arange(nd), decode_ctx_lens=ctxs,
+                                     prefills=prefills)
+    got = harness._bf16_to_f64(d_out.cpu().numpy())
+    err = np.abs(got - want)
+    assert np.all(np.isfinite(got))
+    assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (err.max(), err.mean())
+    np.testing.assert_array_equal(d_kp.cpu().numpy().view(np.uint16), kp)
+    np.testing.assert_array_equal(d_vp.cpu().numpy().view(np.uint16), vp)
+    # the same chunks through the multi-layer iteration call
+    d_out2 = torch.zeros_like(d_out)
+    d_kp2, d_vp2 = t(kp0), t(vp0)
+    ctx.iteration(desc, [ctx.make_bufs(d_q, d_k, d_v, d_kp2, d_vp2, d_out2)])
+    np.testing.assert_array_equal(d_out2.cpu().numpy(), d_out.cpu().numpy())
+    ctx.close()
+
+
+def test_two_chunks_of_one_sequence_rejected():
+    from paper_2609_38386_gb300 import MxError
+    case = Case(16, [40], chunk_start=10, p_t=20, seed=2)
+    ctx = case.make_context()
+    d = case.device_inputs()
+    bad = ctx.make_desc(decode_seq_ids=[0], decode_ctx_lens=[40], page_table=d["page_table"],
+                        slots=d["slots"], prefills=[(1, 10, 20), (1, 30, 5)])   # one sequence twice
+    with pytest.raises(MxError, match="EINVAL"):
+        ctx.mixed_attention(bad, ctx.make_bufs(d["q"], d["k"], d["v"], d["k_pool"], d["v_pool"], d["out"]))
+    ctx.close()

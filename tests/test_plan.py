@@ -20,7 +20,7 @@ def _decode_items(items):
     for x, y, z, w in items.astype(np.int64):
         ux = int(x) & 0xFFFFFFFF
         if ux & 0xF == 0:
-            pre.append(dict(t=y & 0xFFFF, hq=y >> 16, s=z & 0xFFFF, ns=z >> 16, base=int(w)))
+            pre.append(dict(f=ux >> 4, t=y & 0xFFFF, hq=y >> 16, s=z & 0xFFFF, ns=z >> 16, base=int(w)))
         else:
             assert ux & 0xF == 1, hex(ux)
             dec.append(dict(h=(ux >> 4) & 0x7F, s=(ux >> 11) & 0xFFF, len=(ux >> 23) * 16,
@@ -37,8 +37,12 @@ def _plan(hq, ctxs, cs=0, p=0, sms=152, **kw):
                      prefill_seq_id=nd if p else -1, chunk_start=cs, p_t=p, num_sms=sms, **kw)
 
 
-def _check(plan, hq, ctxs, cs, p):
+def _check(plan, hq, ctxs, cs, p, chunks=None):
+    """chunks: [(chunk_start, p_t), ...] for several prefill chunks (else
+    the single chunk cs, p)."""
     hkv = 8
+    if chunks is None:
+        chunks = [(cs, p)] if p else []
     items = plan["items"]
     assert plan["n_items"] == len(items)
     pre, dec = _decode_items(items)
@@ -47,23 +51,25 @@ def _check(plan, hq, ctxs, cs, p):
     # splits, longest first
     kinds = [(int(x) & 0xF) for x in items[:, 0]]
     assert kinds == sorted(kinds)
-    n_qt = -(-p // TILE)
-    n_a = -(-cs // TILE)
-    tiles = [(n_a + d["t"] + 1) * (d["s"] + 1) // d["ns"] - (n_a + d["t"] + 1) * d["s"] // d["ns"]
-             for d in pre]
+    n_a = [-(-c // TILE) for c, _ in chunks]
+    tiles = [(n_a[d["f"]] + d["t"] + 1) * (d["s"] + 1) // d["ns"] -
+             (n_a[d["f"]] + d["t"] + 1) * d["s"] // d["ns"] for d in pre]
     assert all(a >= b for a, b in zip(tiles, tiles[1:]))
 
-    # prefill: each (tile, head) split into pieces that partition its key tiles
+    # prefill: each (chunk, tile, head) split into pieces that partition its
+    # key tiles
     seen = {}
     for d in pre:
-        seen.setdefault((d["t"], d["hq"]), []).append(d)
-    assert set(seen) == {(t, h) for t in range(n_qt) for h in range(hq)}
+        seen.setdefault((d["f"], d["t"], d["hq"]), []).append(d)
+    assert set(seen) == {(f, t, h) for f, (_, p_) in enumerate(chunks)
+                         for t in range(-(-p_ // TILE)) for h in range(hq)}
     bases = []
-    for (t, h), ps in seen.items():
+    for (f, t, h), ps in seen.items():
+        cs, p = chunks[f]
         ns = ps[0]["ns"]
         assert sorted(x["s"] for x in ps) == list(range(ns))
         assert len({x["base"] for x in ps}) == 1
-        n_t = n_a + t + 1
+        n_t = n_a[f] + t + 1
         # the key tiles reach the tile's last row (absolute position); one
         # more, fully masked, only for a ragged last tile whose rows end in
         # the key tile before
@@ -146,6 +152,46 @@ def test_random_iterations(seed):
     kw = dict(split_keys=int(rng.choice([0, 128, 512, 2048])), piece_tiles=int(rng.choice([0, 1, 3, 48])),
               pdl=int(rng.choice([0, 1, 2])))
     _check(_plan(hq, ctxs, cs, p, sms=int(rng.choice([152, 148, 8])), **kw), hq, ctxs, cs, p)
+
+
+MULTI = [
+    # hq, decode contexts, [(chunk_start, p_t), ...]
+    (16, [300, 40], [(0, 100), (256, 200), (7000, 1)]),
+    (32, [], [(128, 128), (77, 300)]),
+    (64, [5000] * 4, [(1000, 300), (0, 4096), (6000, 200), (10, 10)]),
+    (16, [1, 2, 3], [(4096, 256)] + [(c, 17) for c in range(0, 15 * 500, 500)]),
+]
+
+
+def _plan_multi(hq, ctxs, chunks, sms=152, **kw):
+    nd, npf = len(ctxs), len(chunks)
+    n_tok = nd + sum(p for _, p in chunks)
+    max_pages = (max([c + 1 for c in ctxs] + [c + p for c, p in chunks] + [1]) + PAGE - 1) // PAGE
+    return plan_work(num_q_heads=hq, num_kv_heads=8, num_pages=100000, num_seqs=nd + npf,
+                     max_pages_per_seq=max_pages, max_tokens=n_tok, max_decodes=max(nd, 1),
+                     decode_seq_ids=list(range(nd)), decode_ctx_lens=ctxs,
+                     prefills=[(nd + f, c, p) for f, (c, p) in enumerate(chunks)], num_sms=sms, **kw)
+
+
+@pytest.mark.parametrize("hq,ctxs,chunks", MULTI)
+@pytest.mark.parametrize("piece", [0, 3])
+def test_several_chunks_cover_every_key_tile_once(hq, ctxs, chunks, piece):
+    _check(_plan_multi(hq, ctxs, chunks, piece_tiles=piece), hq, ctxs, 0, 0, chunks=chunks)
+
+
+def test_several_chunks_rejections():
+    base = dict(num_q_heads=16, num_pages=1000, num_seqs=4, max_pages_per_seq=64, max_tokens=600,
+                max_decodes=1, decode_seq_ids=[0], decode_ctx_lens=[5])
+    with pytest.raises(MxError, match="EINVAL"):         # two chunks of one sequence
+        plan_work(prefills=[(1, 0, 10), (1, 10, 10)], **base)
+    with pytest.raises(MxError, match="EINVAL"):         # an empty chunk
+        plan_work(prefills=[(1, 0, 0)], **base)
+    with pytest.raises(MxError, match="EINVAL"):         # both forms at once
+        plan_work(prefills=[(1, 0, 10)], prefill_seq_id=2, p_t=5, **base)
+    with pytest.raises(MxError, match="ECAPACITY"):      # more tokens than max_tokens
+        plan_work(prefills=[(1, 0, 300), (2, 0, 300)], **base)
+    with pytest.raises(MxError, match="EINVAL"):         # more than 16 chunks
+        plan_work(**dict(base, num_seqs=40), prefills=[(1 + f, 0, 1) for f in range(17)])
 
 
 def test_options_are_honoured():
