@@ -364,6 +364,72 @@ def independent_layers_measure(w, steps, ws, device):
             "note": "MX_OPT_PDL=2: consecutive layers overlap (valid only for independent layers)"}
 
 
+def several_chunks_measure(cfg, peaks, device, layers=28, reps=10):
+    """Several prompts' chunks in one iteration (four 512-token chunks of
+    four prompts at positions 1024/3072/5120/7168, plus the sweep's 32
+    decodes) against the same decodes with one 2048-token chunk at 4096:
+    device us per 28-layer iteration and the fraction of each iteration's
+    roofline (the slower of its flops at the tensor peak and its bytes at
+    the HBM peak)."""
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2609_38386_gb300 import Context
+    from synth import device as sdev
+    from synth import workload as wl
+    g = cfg.geom
+    it0 = [it for it in cfg.iterations() if it.chunk_size == 0][0]
+    ctxs = [int(c) for c in it0.decode_ctx_lens]
+    nd, npf, plen = len(ctxs), 4, 8192
+    lay = wl.make_layout(g, [c + 1 for c in ctxs] + [plen] * npf, seed=cfg.seed + 991)
+    ps = g.page_size
+    pt_d = torch.from_numpy(lay.page_table).to(device)
+    variants = {"four_512": [(nd + f, 1024 + 2048 * f, 512) for f in range(npf)],
+                "one_2048": [(nd, 4096, 2048)]}
+    n_tok = nd + 2048
+    ctx = Context(num_q_heads=g.hq, num_kv_heads=g.hkv, num_pages=lay.num_pages, num_seqs=lay.num_seqs,
+                  max_pages_per_seq=lay.max_pages, max_tokens=n_tok, max_decodes=nd, device=device.index or 0)
+    bufs, keep = [], []
+    for l in range(layers):
+        t = {}
+        for name, shape, kind in (("q", (n_tok, g.hq, g.head_dim), 0), ("k", (n_tok, g.hkv, g.head_dim), 1),
+                                  ("v", (n_tok, g.hkv, g.head_dim), 2), ("kp", lay.pool_shape(), 3),
+                                  ("vp", lay.pool_shape(), 4)):
+            t[name] = torch.empty(shape, dtype=torch.int16, device=device)
+            sdev.fill_(t[name], synth.stream_base(cfg.seed + 991, synth.stream_id(l, kind)))
+        t["o"] = torch.empty((n_tok, g.hq, g.head_dim), dtype=torch.int16, device=device)
+        keep.append(t)
+        bufs.append(ctx.make_bufs(t["q"], t["k"], t["v"], t["kp"], t["vp"], t["o"]))
+    arr = ctx.layer_array(bufs)
+    out = {}
+    for name, pfs in variants.items():
+        slots = [lay.page_table[i, c // ps] * ps + c % ps for i, c in enumerate(ctxs)]
+        B = F = 0
+        for seq, cs, p in pfs:
+            slots += [lay.page_table[seq, (cs + j) // ps] * ps + (cs + j) % ps for j in range(p)]
+            b_, f_ = wl.algorithmic_work(g, wl.IterSpec(0, np.zeros(0, np.int32), np.zeros(0, np.int32),
+                                                        seq, cs, p, p))
+            B, F = B + b_, F + f_
+        b_, f_ = wl.algorithmic_work(g, wl.IterSpec(0, it0.decode_seq_ids, it0.decode_ctx_lens, -1, 0, 0, 0))
+        B, F = (B + b_) * layers, (F + f_) * layers
+        sl_d = torch.from_numpy(np.asarray(slots, np.int32)).to(device)
+        desc = ctx.make_desc(decode_seq_ids=list(range(nd)), decode_ctx_lens=ctxs, page_table=pt_d,
+                             slots=sl_d, prefills=pfs)
+        us = [ctx.iteration(desc, arr) for _ in range(reps + 3)][3:]
+        ctx.sync_status()
+        t_us = float(np.median(us))
+        roof = max(F / (peaks["bf16_tflops_sustained"] * 1e12), B / (peaks["hbm_gbs"] * 1e9)) * 1e6
+        out[name] = {"chunks": [[cs, p] for _, cs, p in pfs], "device_us_p50": t_us,
+                     "roofline_us": roof, "roofline_frac": roof / t_us,
+                     "tokens_per_s": (nd + sum(p for _, _, p in pfs)) / t_us * 1e6}
+    ctx.close()
+    del keep
+    torch.cuda.empty_cache()
+    return dict(out, note="32 decodes U[512,4096] + the chunks, 28 layers with distinct pools; "
+                          "roofline from the measured peaks")
+
+
 # ------------------------------------------------------------- CPU oracle
 def oracle_sample(cfg, which="heavy"):
     """A bounded slice of the workload for the CPU oracle: one layer call of
@@ -712,6 +778,8 @@ def main():
         line["e2e"] = e2e_measure(w, max(1, min(args.steps, 3)), device)
     if not args.profile:
         line["independent_layers"] = independent_layers_measure(w, args.steps, ws, device)
+    if not args.profile and args.config == "qwen3-0.6b-attn-28L-chunk-sweep" and rank == 0:
+        line["several_chunks"] = several_chunks_measure(cfg, peaks, device)
     if rank == 0 and ws == 1 and not args.no_cpu and not args.profile:
         line["cpu_baseline"] = cpu_baseline(cfg)
     if rank == 0:
