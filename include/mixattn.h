@@ -230,10 +230,11 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  * MX_OPT_PREFILL_PIECE_TILES and MX_OPT_PDL (0, 0 and 1 are the defaults).
  * Outputs (host arrays owned by the caller):
  *   items    int32 [max_items][4], n_items records in claim order:
- *     prefill {0, t | hq << 16, s | n_s << 16, partial slot base}: piece s
- *       of n_s of query tile t (chunk rows [128 t, 128 t + 128)) of query
- *       head hq; the tile's n_T = ceil(chunk_start / 128) + t + 1 key tiles
- *       (128 keys each) are split as [s n_T / n_s, (s + 1) n_T / n_s);
+ *     prefill {f << 4, t | hq << 16, s | n_s << 16, partial slot base}:
+ *       piece s of n_s of query tile t (rows [128 t, 128 t + 128) of prefill
+ *       chunk f, in the order of desc->prefills, or 0 for the single chunk)
+ *       of query head hq; the tile's n_T = ceil(chunk_start_f / 128) + t + 1
+ *       key tiles (128 keys each) are split as [s n_T / n_s, (s + 1) n_T / n_s);
  *     decode {1 | h << 4 | s << 11 | (len / 16) << 23, decode index i,
  *       page-table row, cached tokens ctx}: split s of decode i, KV head h,
  *       keys [s len, min((s + 1) len, ctx + 1));
