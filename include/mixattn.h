@@ -237,7 +237,8 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  *       key tiles (128 keys each) are split as [s n_T / n_s, (s + 1) n_T / n_s);
  *     decode {1 | h << 4 | s << 11 | (len / 16) << 23, decode index i,
  *       page-table row, cached tokens ctx}: split s of decode i, KV head h,
- *       keys [s len, min((s + 1) len, ctx + 1));
+ *       keys [s len, min((s + 1) len, ctx + 1)); kind 2 instead of 1 for a
+ *       decode of at most 16 keys (one split, computed exactly in fp32);
  *   decodes  int32 [n_decodes][4]: page-table row, ctx, number of splits,
  *     first partial slot (of head 0; head h uses base + h * splits);
  *   counts   int32 [4]: n_items, prefill items, split_keys, piece_tiles.

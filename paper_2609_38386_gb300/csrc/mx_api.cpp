@@ -432,8 +432,12 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
                        n_prefill + ditems.size(), k.max_items);
     std::stable_sort(ditems.begin(), ditems.end(),
                      [](const DItem &a, const DItem &b) { return a.keys > b.keys; });
-    for (const DItem &x : ditems)
-        items[n++] = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx, x.len);
+    for (const DItem &x : ditems) {
+        int4 code = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx, x.len);
+        if (dec[x.i].ctx + 1 <= kPage)  // at most 16 keys: the exact short path
+            code.x = (int32_t)(((uint32_t)code.x & ~0xFu) | (uint32_t)ITEM_DECODE_SHORT);
+        items[n++] = code;
+    }
 
     out->n_items = n;
     out->n_prefill = n_prefill;

@@ -48,7 +48,7 @@ constexpr uint32_t kTmemCols = 512;
 constexpr int kSBuf = 3;
 constexpr uint32_t kTmemO = kSBuf * 128;
 
-enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1 };
+enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1, ITEM_DECODE_SHORT = 2 };
 
 // Prefill chunks of one iteration (several prompts' chunks may share it).
 constexpr int kMaxPrefills = 16;
@@ -66,6 +66,8 @@ struct PrefillInfo {
 //             partial slot base}: piece s of n_s of query tile t (rows
 //            [128t, 128t+128) of chunk f) of head hq; the tile's key tiles are
 //            split evenly between its n_s pieces.
+//   short decode (at most 16 keys, one split): the decode record with kind
+//            ITEM_DECODE_SHORT;
 //   decode:  {ITEM_DECODE | kv head << 4 | split index << 11 | split
 //             length / 16 << 23, decode index, page-table row, cached tokens}:
 //             split s of decode i covers keys [s * len, (s + 1) * len) of

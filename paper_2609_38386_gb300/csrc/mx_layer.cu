@@ -20,6 +20,7 @@
 //                           query heads of the group at once: a split-KV
 //                           flash-decode whose partial (O, lse) is merged by
 //                           the last-arriving split (no waiting).
+//   ITEM_DECODE_SHORT: a decode of at most 16 keys, exact on CUDA cores.
 // New keys/values are read from the k/v inputs, never from the pages being
 // written in the same launch, so the append needs no ordering.
 #include "mx_internal.h"
@@ -66,6 +67,84 @@ __device__ __forceinline__ void set_abort(const LayerParams &P, Misc *misc)
 }
 
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
+
+// ---------------------------------------------------------------------------
+// A decode of at most 16 keys (fewer than 16 cached tokens), KV head h: exact
+// fp32 attention on the CUDA cores.  With so few keys the bf16 rounding of a
+// single weight of P in the tensor-core path would show in the output.  The
+// scores go through shared memory; cached K/V rows are read from their page,
+// the new key from the k/v inputs (as in the split path), which it appends.
+// ---------------------------------------------------------------------------
+__device__ void decode_short_item(const LayerParams &P, uint8_t *smem, int di, int h, int seq, int n)
+{
+    const int tid = threadIdx.x, nrep = P.n_rep, nk = n + 1;
+    float *ss = reinterpret_cast<float *>(smem);  // [kMaxRep][16] scores (log2 domain)
+    if (tid < 32) {
+        const int slot = P.slots[di];
+        if (slot >= P.num_pages * kPage) {
+            if (tid == 0)
+                flag_error(P, ERR_SLOT);
+        } else if (slot >= 0) {
+            const size_t dst = (((size_t)(slot / kPage) * P.hkv + h) * kPage + slot % kPage) * kHeadDim;
+            const size_t src = ((size_t)di * P.hkv + h) * kHeadDim;
+            const int c = tid & 15;
+            if (tid < 16)
+                reinterpret_cast<uint4 *>(P.k_pool + dst)[c] = __ldg(reinterpret_cast<const uint4 *>(P.k + src) + c);
+            else
+                reinterpret_cast<uint4 *>(P.v_pool + dst)[c] = __ldg(reinterpret_cast<const uint4 *>(P.v + src) + c);
+        }
+    }
+    int pid = -1;
+    if (n > 0) {
+        pid = __ldg(P.page_table + (size_t)seq * P.max_pages);
+        if (pid < 0 || pid >= P.num_pages) {
+            if (tid == 0)
+                flag_error(P, ERR_PAGE);
+            pid = -1;
+        }
+    }
+    const uint16_t *knew = P.k + ((size_t)di * P.hkv + h) * kHeadDim;
+    const uint16_t *vnew = P.v + ((size_t)di * P.hkv + h) * kHeadDim;
+    const size_t pbase = ((size_t)(pid < 0 ? 0 : pid) * P.hkv + h) * kPage * kHeadDim;
+    if (tid < nrep * kPage) {
+        const int q = tid / kPage, k = tid % kPage;
+        float s = neg_inf();
+        if (k < nk && (k == n || pid >= 0)) {
+            const uint4 *qr = reinterpret_cast<const uint4 *>(P.q + ((size_t)di * P.hq + h * nrep + q) * kHeadDim);
+            const uint4 *kr = reinterpret_cast<const uint4 *>(k < n ? P.k_pool + pbase + (size_t)k * kHeadDim : knew);
+            float acc = 0.f;
+#pragma unroll 4
+            for (int c = 0; c < 16; ++c) {
+                const uint4 a = __ldg(qr + c), b = __ldg(kr + c);
+                const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    acc += bf16lo(aw[e]) * bf16lo(bw[e]) + bf16hi(aw[e]) * bf16hi(bw[e]);
+            }
+            s = acc * P.scale_log2;
+        }
+        ss[q * kPage + k] = s;
+    }
+    __syncthreads();
+    for (int e = tid; e < nrep * kHeadDim; e += kThreads) {
+        const int q = e / kHeadDim, d = e % kHeadDim;
+        float m = neg_inf();
+        for (int k = 0; k < nk; ++k)
+            m = fmaxf(m, ss[q * kPage + k]);
+        float l = 0.f, o = 0.f;
+        for (int k = 0; k < nk; ++k) {
+            const float sk = ss[q * kPage + k];
+            if (sk == neg_inf())
+                continue;
+            const float pk = ex2(sk - m);
+            const uint16_t vb = k < n ? P.v_pool[pbase + (size_t)k * kHeadDim + d] : vnew[d];
+            l += pk;
+            o += pk * __uint_as_float((uint32_t)vb << 16);
+        }
+        __nv_bfloat16 b = __float2bfloat16_rn(o / l);
+        P.out[((size_t)di * P.hq + h * nrep + q) * kHeadDim + d] = *reinterpret_cast<uint16_t *>(&b);
+    }
+}
 
 // ---------------------------------------------------------------------------
 // Decode split: keys [k_lo, k_hi) of decode di, KV head h.
@@ -975,9 +1054,10 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     }
     if (tid >= 64 && tid < 64 + P.n_prefills)
         misc->pre[tid - 64] = P.pre[tid - 64];
-    // Consecutive launches use alternate workspace sets, and the launch two
-    // back has completed before this one was launched (see the end of the
-    // kernel), so work starts at once, beside the previous layer's tail.
+    // Consecutive launches use the workspace sets in turn, and the launch
+    // that last used this one's set has completed before this one was
+    // launched (see the end of the kernel), so work starts at once, beside
+    // the previous layer's tail.
     if (tid == 0) {
         misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
         // Fault injection for the bounded waits: the chosen block waits on a
@@ -1026,6 +1106,8 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
                 merge_ns = ns;
                 merge_f = f;
             }
+        } else if ((it.x & 0xF) == ITEM_DECODE_SHORT) {
+            decode_short_item(P, smem, it.y, (int)(((uint32_t)it.x >> 4) & 0x7Fu), it.z, it.w);
         } else {
             const uint32_t dx = (uint32_t)it.x;
             decode_item(P, smem, misc, it.y, (int)((dx >> 4) & 0x7Fu), (int)((dx >> 11) & 0xFFFu), it.z, it.w,

@@ -254,6 +254,9 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
         const int kc = dec[c.y].ctx + 1 - (dec[c.y].n_splits - 1) * split;
         return ka > kc;
     });
+    for (int x = tail0; x < n; ++x)   // at most 16 keys: the exact short path
+        if (dec[items[x].y].ctx + 1 <= kPage)
+            items[x].x = (int32_t)(((uint32_t)items[x].x & ~0xFu) | (uint32_t)ITEM_DECODE_SHORT);
 
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess)

@@ -22,7 +22,9 @@ def _decode_items(items):
         if ux & 0xF == 0:
             pre.append(dict(f=ux >> 4, t=y & 0xFFFF, hq=y >> 16, s=z & 0xFFFF, ns=z >> 16, base=int(w)))
         else:
-            assert ux & 0xF == 1, hex(ux)
+            # 1: a split; 2: a decode of at most 16 keys (exact short path)
+            assert ux & 0xF in (1, 2), hex(ux)
+            assert ux & 0xF == 1 or int(w) + 1 <= PAGE
             dec.append(dict(h=(ux >> 4) & 0x7F, s=(ux >> 11) & 0xFFF, len=(ux >> 23) * 16,
                             i=int(y), row=int(z), ctx=int(w)))
     return pre, dec
