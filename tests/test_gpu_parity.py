@@ -29,7 +29,7 @@ def test_small_config_full_parity():
     _ok(case.check(res))
 
 
-@pytest.mark.parametrize("ctx", [[0], [1, 15, 16, 17], [5, 300, 1023, 1024, 2049],
+@pytest.mark.parametrize("ctx", [[0], [1, 15, 16, 17], list(range(16)), [5, 300, 1023, 1024, 2049],
                                  [4095, 4096, 7000]])
 @pytest.mark.parametrize("hq", [16, 64])
 def test_decode_only(ctx, hq):
