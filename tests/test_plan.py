@@ -25,7 +25,7 @@ def _decode_items(items):
             # 1: a split; 2: a decode of at most 16 keys (exact short path)
             assert ux & 0xF in (1, 2), hex(ux)
             assert ux & 0xF == 1 or int(w) + 1 <= PAGE
-            dec.append(dict(h=(ux >> 4) & 0x7F, s=(ux >> 11) & 0xFFF, len=(ux >> 23) * 16,
+            dec.append(dict(kind=ux & 0xF, h=(ux >> 4) & 0x7F, s=(ux >> 11) & 0xFFF, len=(ux >> 23) * 16,
                             i=int(y), row=int(z), ctx=int(w)))
     return pre, dec
 
@@ -96,6 +96,7 @@ def _check(plan, hq, ctxs, cs, p, chunks=None):
     seen = {}
     for d in dec:
         assert d["row"] == d["i"] and d["ctx"] == ctxs[d["i"]]
+        assert d["kind"] == (2 if ctxs[d["i"]] + 1 <= PAGE else 1)   # the exact short path
         assert d["len"] % PAGE == 0 and 0 < d["len"] <= 4096
         seen.setdefault((d["i"], d["h"]), []).append(d)
     assert set(seen) == {(i, h) for i in range(len(ctxs)) for h in range(hkv)}
