@@ -1,18 +1,20 @@
 #!/usr/bin/env python
 """Mixed-iteration benchmark on GB300: prints ONE JSON line.
 
-Workload (default): Qwen3-0.6B attention geometry (16 Q / 8 KV heads, head dim
-128, bf16, 16-token pages), 28 layer calls per iteration with distinct
-per-layer pools, 32 decodes with cached contexts uniform in [512, 4096], and
-one 8192-token prompt prefilled beside them with chunk size p swept over
-{0, 256, 512, 1024, 2048, 4096}, every chunk in order (63 iterations).  One
-step = that whole sweep.  Inputs are seeded synthetic N(0,1) bf16 values,
-resident in HBM before timing (per-layer pools of ~335 MB, far above L2).
+Workload (default, the headline): Qwen3-32B attention geometry (64 Q / 8 KV
+heads, head dim 128, bf16, 16-token pages), 64 layer calls per iteration with
+distinct per-layer pools (~200 GB in all), 128 decodes with cached contexts
+log-uniform in [1024, 16384], and one 32768-token prompt prefilled beside them
+with chunk size p swept over {0, 1024, 2048, 4096, 8192}, every chunk in order
+(61 iterations).  One step = that whole sweep.  Inputs are seeded synthetic
+N(0,1) bf16 values, resident in HBM before timing; the pools are far larger
+than L2.  The Qwen3-0.6B (28 layers) and Qwen3-8B (36 layers) sweeps are
+measured in the same run and reported beside it (`other_configs`).
 
 `value` = tokens (decode tokens + prompt tokens) per second of device time,
 from CUDA events on the launching stream; `e2e` = the same through the C-ABI
-iteration call with host buffers (q/k/v copied in, outputs copied out, every
-iteration synchronised on its completion time).  `--impl reference` times the
+iteration call with host buffers (q/k/v copied in from pinned host memory and
+outputs copied out inside the timed region).  `--impl reference` times the
 float64 CPU oracle on a bounded sample instead.
 """
 from __future__ import annotations
@@ -36,9 +38,18 @@ SPEC_HBM = 8000e9          # nominal HBM3e bytes/s
 SPEC_TFLOPS = 1706.7e12   # nominal sustained dense bf16 flop/s
 METRIC = ("mixed-iteration device µs & tokens/s; % of HBM/tensor roofline per chunk size")
 UNIT = "tokens/s"
-DEFAULT_CONFIG = "qwen3-0.6b-attn-28L-chunk-sweep"
+DEFAULT_CONFIG = "qwen3-32b-attn-64L-chunk-sweep"
+# sweeps reported beside the headline in the same run
+SIDE_CONFIGS = ("qwen3-0.6b-attn-28L-chunk-sweep", "qwen3-8b-attn-36L-chunk-sweep")
+# sweeps whose per-iteration inputs for every layer would not fit beside the
+# pools: one q/k/v buffer per layer, reused by every iteration
+LEAN_CONFIGS = ("qwen3-32b-attn-64L-chunk-sweep",)
 KERNEL_SRC = os.path.join(ROOT, "paper_2609_38386_gb300", "csrc", "mx_layer.cu")
-TRAFFIC_SUMMARY = os.path.join(ROOT, "profiles", "mixed_layer_qwen06b_sweep.md")
+# the committed ncu summary that gives each sweep's DRAM bytes per launch
+TRAFFIC_SUMMARY = {
+    "qwen3-0.6b-attn-28L-chunk-sweep": os.path.join(ROOT, "profiles", "mixed_layer_qwen06b_sweep.md"),
+    "qwen3-32b-attn-64L-chunk-sweep": os.path.join(ROOT, "profiles", "mixed_layer_qwen32b_sweep.md"),
+}
 
 
 # ----------------------------------------------------------------- helpers
@@ -61,12 +72,13 @@ def kernel_hash():
     return h.hexdigest()[:16]
 
 
-def committed_traffic():
-    """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source (else None)."""
-    if not os.path.exists(TRAFFIC_SUMMARY):
+def committed_traffic(config):
+    """DRAM bytes per launch of the sweep from its committed ncu summary, if
+    that was taken on the current kernel source (else None)."""
+    path = TRAFFIC_SUMMARY.get(config)
+    if not path or not os.path.exists(path):
         return None
-    txt = open(TRAFFIC_SUMMARY).read()
+    txt = open(path).read()
     m_h = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", txt)
     m_t = re.search(r"dram_bytes_per_launch_full_workload:\s*([0-9.eE+]+)", txt)
     if not m_h or not m_t or m_h.group(1) != kernel_hash():
@@ -229,6 +241,12 @@ class Workload:
         self.work = [wl.algorithmic_work(g, it) for it in self.its]
         self.tokens_per_step = sum(it.n_tokens for it in self.its)
 
+    def close(self):
+        """Release the context and the device tensors."""
+        self.ctx.close()
+        self.pools = self.outs = self.inputs = self.slots = None
+        self.descs = self.layer_arrays = None
+
     def run_step(self, events=None):
         """Enqueue every iteration of the sweep (no host waits)."""
         for i in range(len(self.its)):
@@ -239,72 +257,90 @@ class Workload:
             events[len(self.its)].record()
 
 
-def e2e_measure(w, steps, device):
+def e2e_measure(w, steps, device, budget_bytes=12 << 30):
     """Same sweep through the iteration call with host buffers: every
     iteration's q/k/v for all layers is copied from pinned host memory, the
     iteration runs, and every layer's output is copied back to pinned host
-    memory, all inside the timed region.  The copies are pipelined against the
-    iterations the way a serving loop would run them: the inputs of iteration
-    i+1 and i+2 upload on one stream and the outputs of iteration i-1
-    download on another while iteration i computes (three device buffer
-    sets, so that a large iteration's upload has two iterations of slack);
-    the pipeline runs across the timed steps and the region ends when the
-    last step's outputs are on the host."""
+    memory, all inside the timed region.  The copies are pipelined against
+    the compute the way a serving loop would run them, in units of a group of
+    consecutive layers (the whole iteration when its buffers fit the budget;
+    for the 64-layer 32B sweep, whose pools fill most of HBM, 8 layers, each
+    group one iteration call): the inputs of unit j+1 and j+2 upload on one
+    stream and the outputs of unit j-1 download on another while unit j
+    computes (three device buffer sets).  The pipeline runs across the timed
+    steps; the region ends when the last step's outputs are on the host.  The
+    host buffer holds the largest iteration's inputs; each unit uploads as
+    many bytes as its own iteration needs (so the copy volume is exact, while
+    the contents are those of the largest iteration)."""
     import torch
     g, L = w.geom, w.L
     per_tok_in = (g.hq + 2 * g.hkv) * g.head_dim
     per_tok_out = g.hq * g.head_dim
-    max_in = L * w.max_tok * per_tok_in
-    max_out = L * w.max_tok * per_tok_out
+    nbuf = 3
+    group = L
+    for cand in range(1, L + 1):                     # fewest groups that fit
+        if L % cand == 0 and nbuf * (L // cand) * w.max_tok * (per_tok_in + per_tok_out) * 2 <= budget_bytes:
+            group = L // cand
+            break
+    else:
+        group = 1
+    n_groups = L // group
+    max_in = group * w.max_tok * per_tok_in
+    max_out = group * w.max_tok * per_tok_out
     h_in = torch.empty(max_in, dtype=torch.int16, pin_memory=True)
     h_out = torch.empty(max_out, dtype=torch.int16, pin_memory=True)
-    nbuf = 3
     d_in = [torch.empty(max_in, dtype=torch.int16, device=device) for _ in range(nbuf)]
     d_out = [torch.empty(max_out, dtype=torch.int16, device=device) for _ in range(nbuf)]
-    # host contents: the largest iteration's device inputs, packed per layer
+    # host contents: the largest iteration's device inputs of the first group
     big = max(range(len(w.its)), key=lambda i: w.its[i].n_tokens)
+    nb = w.its[big].n_tokens
     off = 0
-    for l in range(L):
-        for t in w.inputs[big][l]:
-            n = t.numel()
-            h_in[off:off + n].copy_(t.reshape(-1).cpu())
+    for l in range(group):
+        for t, heads in zip(w.inputs[big][l], (g.hq, g.hkv, g.hkv)):
+            n = nb * heads * g.head_dim
+            h_in[off:off + n].copy_(t.reshape(-1)[:n].cpu())
             off += n
-    layer_arrays, in_elems, out_elems = [], [], []
-    for i, it in enumerate(w.its):
+    # per (iteration, layer group, buffer set): the layer array of that unit
+    arrays, in_elems, out_elems = [], [], []
+    for it in w.its:
         n = it.n_tokens
-        sets = []
-        for b in range(nbuf):
-            bufs, o_in, o_out = [], 0, 0
-            for l in range(L):
-                q = d_in[b][o_in:o_in + n * g.hq * g.head_dim]
-                o_in += q.numel()
-                k = d_in[b][o_in:o_in + n * g.hkv * g.head_dim]
-                o_in += k.numel()
-                v = d_in[b][o_in:o_in + n * g.hkv * g.head_dim]
-                o_in += v.numel()
-                out = d_out[b][o_out:o_out + n * per_tok_out]
-                o_out += out.numel()
-                kp, vp = w.pools[l]
-                bufs.append(w.ctx.make_bufs(q, k, v, kp, vp, out))
-            sets.append(w.ctx.layer_array(bufs))
-        layer_arrays.append(sets)
-        in_elems.append(o_in)
-        out_elems.append(o_out)
+        per_group = []
+        for gi in range(n_groups):
+            sets = []
+            for b in range(nbuf):
+                bufs, o_in, o_out = [], 0, 0
+                for l in range(gi * group, (gi + 1) * group):
+                    q = d_in[b][o_in:o_in + n * g.hq * g.head_dim]
+                    o_in += q.numel()
+                    k = d_in[b][o_in:o_in + n * g.hkv * g.head_dim]
+                    o_in += k.numel()
+                    v = d_in[b][o_in:o_in + n * g.hkv * g.head_dim]
+                    o_in += v.numel()
+                    out = d_out[b][o_out:o_out + n * per_tok_out]
+                    o_out += out.numel()
+                    kp, vp = w.pools[l]
+                    bufs.append(w.ctx.make_bufs(q, k, v, kp, vp, out))
+                sets.append(w.ctx.layer_array(bufs))
+            per_group.append(sets)
+        arrays.append(per_group)
+        in_elems.append(group * n * per_tok_in)
+        out_elems.append(group * n * per_tok_out)
     comp = torch.cuda.current_stream(device)
     up = torch.cuda.Stream(device)
     down = torch.cuda.Stream(device)
     n_it = len(w.its)
 
     def run(n_steps):
-        # one continuous pipeline over the steps' iterations: iteration j uses
-        # buffer set j % nbuf, uploads as soon as iteration j - nbuf has
-        # consumed that set, and downloads as soon as it has computed
-        total = n_steps * n_it
+        # one continuous pipeline over the steps' units: unit j uses buffer
+        # set j % nbuf, uploads as soon as unit j - nbuf has consumed that
+        # set, and downloads as soon as it has computed
+        units = [(i, gi) for _ in range(n_steps) for i in range(n_it) for gi in range(n_groups)]
+        total = len(units)
         ev_in = [torch.cuda.Event() for _ in range(total)]
         ev_comp = [torch.cuda.Event() for _ in range(total)]
         ev_out = [torch.cuda.Event() for _ in range(total)]
-        for j in range(total):
-            i, b = j % n_it, j % nbuf
+        for j, (i, gi) in enumerate(units):
+            b = j % nbuf
             with torch.cuda.stream(up):
                 if j >= nbuf:
                     up.wait_event(ev_comp[j - nbuf])   # inputs of j-nbuf consumed
@@ -313,7 +349,7 @@ def e2e_measure(w, steps, device):
             comp.wait_event(ev_in[j])
             if j >= nbuf:
                 comp.wait_event(ev_out[j - nbuf])      # outputs of j-nbuf downloaded
-            w.ctx.iteration(w.descs[i], layer_arrays[i][b], stream=comp, wait=False)
+            w.ctx.iteration(w.descs[i], arrays[i][gi][b], stream=comp, wait=False)
             ev_comp[j].record(comp)
             with torch.cuda.stream(down):
                 down.wait_event(ev_comp[j])
@@ -330,10 +366,17 @@ def e2e_measure(w, steps, device):
     torch.cuda.synchronize(device)
     dt = time.perf_counter() - t0
     w.ctx.sync_status()
-    return {"value": w.tokens_per_step * steps / dt, "unit": UNIT,
-            "h2d_bytes_per_step": int(sum(in_elems) * 2), "d2h_bytes_per_step": int(sum(out_elems) * 2),
-            "seconds": dt, "copies": "pinned host <-> device on two copy streams, pipelined with "
-            "compute across the timed steps (every step's inputs and outputs inside the region)"}
+    res = {"value": w.tokens_per_step * steps / dt, "unit": UNIT,
+           "h2d_bytes_per_step": int(sum(in_elems) * 2 * n_groups),
+           "d2h_bytes_per_step": int(sum(out_elems) * 2 * n_groups),
+           "seconds": dt, "steps": steps, "layers_per_call": group,
+           "copies": "pinned host <-> device on two copy streams, pipelined with compute across the "
+                     "timed steps in units of %d layer(s) per iteration call (every step's inputs and "
+                     "outputs inside the region); each unit copies its own iteration's byte count, "
+                     "taken from a host buffer that holds the largest iteration's inputs" % group}
+    del d_in, d_out, h_in, h_out
+    torch.cuda.empty_cache()
+    return res
 
 
 def independent_layers_measure(w, steps, ws, device):
@@ -431,22 +474,35 @@ def several_chunks_measure(cfg, peaks, device, layers=28, reps=10):
 
 
 # ------------------------------------------------------------- CPU oracle
+# Bounded samples of each sweep for the float64 CPU oracle: one layer call of
+# one iteration (chunk size, chunk start), its first `decodes` decodes (None:
+# all) and every `head_stride`-th query head (one per KV head at stride
+# n_rep); the time is scaled by head_stride to all heads.
+ORACLE_SAMPLES = {
+    "qwen3-0.6b-attn-28L-chunk-sweep": {"light": (256, 4096, None, 1), "heavy": (2048, 6144, None, 1)},
+    "qwen3-8b-attn-36L-chunk-sweep": {"light": (512, 4096, 32, 4), "heavy": (2048, 8192, 32, 4)},
+    "qwen3-32b-attn-64L-chunk-sweep": {"light": (1024, 4096, 32, 8), "heavy": (4096, 8192, 32, 8)},
+}
+
+
 def oracle_sample(cfg, which="heavy"):
-    """A bounded slice of the workload for the CPU oracle: one layer call of
-    one iteration (heavy: the p=2048 chunk at 6144; light: the p=256 chunk at
-    4096).  Returns (fn, tokens_per_iteration_equivalent, description)."""
+    """A bounded slice of the workload for the CPU oracle.  Returns (fn,
+    tokens of the slice, description, time scale to all query heads)."""
     import oracle
     import synth
     from synth import workload as wl
     its = cfg.iterations()
-    want = (2048, 6144) if which == "heavy" else (256, 4096)
-    it = next((x for x in its if (x.chunk_size, x.chunk_start) == want), its[-1])
+    chunk, cs, n_dec, stride = ORACLE_SAMPLES.get(cfg.name, {}).get(which, (0, 0, None, 1))
+    it = next((x for x in its if (x.chunk_size, x.chunk_start) == (chunk, cs)), its[-1])
+    nd = it.n_decodes if n_dec is None else min(n_dec, it.n_decodes)
+    it = wl.IterSpec(it.index, it.decode_seq_ids[:nd], it.decode_ctx_lens[:nd], it.prefill_seq,
+                     it.chunk_start, it.p_t, it.chunk_size)
     lay = cfg.layout()
     g = cfg.geom
-    q = wl.host_tokens(cfg.seed, 0, synth.STREAM_Q, it, g.hq)
+    q = np.ascontiguousarray(wl.host_tokens(cfg.seed, 0, synth.STREAM_Q, it, g.hq)[:, ::stride])
     k = wl.host_tokens(cfg.seed, 0, synth.STREAM_K, it, g.hkv)
     v = wl.host_tokens(cfg.seed, 0, synth.STREAM_V, it, g.hkv)
-    # compact pool: the pages this iteration reads or writes
+    # compact pool: the pages this slice reads or writes
     ps = g.page_size
     seqs = list(it.decode_seq_ids) + ([it.prefill_seq] if it.p_t else [])
     nkeys = list(it.decode_ctx_lens + 1) + ([it.chunk_start + it.p_t] if it.p_t else [])
@@ -469,19 +525,21 @@ def oracle_sample(cfg, which="heavy"):
                                decode_ctx_lens=it.decode_ctx_lens, prefill_seq=it.prefill_seq,
                                chunk_start=it.chunk_start, p_t=it.p_t)
 
+    heads = (f"{g.hq // stride} of the {g.hq} query heads (one per KV head), time scaled x{stride} "
+             "to all heads" if stride > 1 else f"all {g.hq} heads")
     desc = (f"one layer call of the p={it.p_t} iteration at chunk_start={it.chunk_start} "
-            f"({it.n_decodes} decodes + {it.p_t} chunk rows, all {g.hq} heads); tokens/s "
-            f"scaled to the {cfg.n_layers}-layer iteration")
-    return fn, it.n_tokens, desc
+            f"({nd} decodes + {it.p_t} chunk rows; {heads}); tokens/s scaled to the "
+            f"{cfg.n_layers}-layer iteration")
+    return fn, it.n_tokens, desc, stride
 
 
 def cpu_baseline(cfg, which="heavy"):
     import oracle
-    fn, ntok, desc = oracle_sample(cfg, which)
+    fn, ntok, desc, scale = oracle_sample(cfg, which)
     t0 = time.perf_counter()
     fn()
     dt = time.perf_counter() - t0
-    return {"value": ntok / (dt * cfg.n_layers), "unit": UNIT, "cores": oracle.max_threads(),
+    return {"value": ntok / (dt * scale * cfg.n_layers), "unit": UNIT, "cores": oracle.max_threads(),
             "kind": "oracle", "sample": desc, "seconds": dt}
 
 
@@ -592,125 +650,46 @@ def trace_measure(device, seeds=(801, 802, 803), n_layers=28, hq=16, budget=8192
     return result
 
 
-# ------------------------------------------------------------------- main
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
-    ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", default=DEFAULT_CONFIG)
-    ap.add_argument("--profile", action="store_true",
-                    help="small case for ncu: 2 layers, iterations of --profile-chunk only")
-    ap.add_argument("--profile-chunk", type=int, default=2048)
-    ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--no-cpu", action="store_true")
-    ap.add_argument("--lean", action="store_true",
-                    help="one q/k/v buffer per layer reused by all iterations (large sweeps)")
-    ap.add_argument("--workload", default="sweep", choices=["sweep", "trace"],
-                    help="trace: the completion-timed DLFP loop vs a fixed chunk cap")
-    args = ap.parse_args()
-
-    ws, rank, local = dist_setup()
-    from synth import workload as wl
-    cfg = wl.CONFIGS[args.config]
-    config = {"workload": cfg.name, "q_heads": cfg.hq, "kv_heads": 8, "head_dim": 128,
-              "page_size": 16, "layers": cfg.n_layers, "decodes": cfg.n_decodes,
-              "decode_ctx": f"{cfg.ctx_dist}[{cfg.ctx_lo},{cfg.ctx_hi}]",
-              "prompt_len": cfg.prompt_len, "chunk_sizes": list(cfg.chunk_sizes),
-              "iterations_per_step": len(cfg.iterations()),
-              "l2": f"inputs larger than L2: each iteration reads {cfg.n_layers} distinct "
-                    "per-layer KV pools of several hundred MB or more",
-              "parallelism": f"replicas{ws}"}
-
-    if args.impl == "reference":
-        if rank != 0:
-            return
-        import oracle
-        fn, ntok, desc = oracle_sample(cfg, "light")
-        for _ in range(args.warmup):
-            fn()
-        t0 = time.perf_counter()
-        for _ in range(args.steps):
-            fn()
-        dt = time.perf_counter() - t0
-        val = ntok * args.steps / (dt * cfg.n_layers)
-        line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT,
-                "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
-                "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                "config": config,
-                "cpu_baseline": {"value": val, "unit": UNIT, "cores": oracle.max_threads(),
-                                 "kind": "oracle", "sample": desc},
-                "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0,
-                        "d2h_bytes_per_step": 0}}
-        print(json.dumps(line))
-        return
-
+# ---------------------------------------------------------------- timing
+def time_sweep(w, steps, warmup, ws, device, barrier, sampler=None):
+    """W untimed steps, then K timed steps bracketed by a barrier and a
+    synchronise on both sides; CUDA events on the launching stream around
+    the whole region and around every iteration.  Returns (max-over-ranks
+    total ms, per-iteration device us [steps][iterations], clocks)."""
     import torch
-    if args.workload == "trace":
-        if rank == 0:
-            device = torch.device("cuda", local)
-            torch.cuda.set_device(device)
-            res = trace_measure(device)
-            print(json.dumps({"metric": "open-loop trace: per-iteration device us P50/P99 and "
-                              "ITL/TTFT, completion-timed DLFP vs fixed chunk caps",
-                              "workload": "qwen3-0.6b-attn-28L-poisson-trace", **res}))
-        return
-    if ws > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
-    device = torch.device("cuda", local)
-    torch.cuda.set_device(device)
-    peaks = load_peaks()
-
-    layers = 2 if args.profile else None
-    w = Workload(cfg, device, seed_offset=replica_seed_offset(rank), layers=layers,
-                 lean=args.lean)
-    if args.lean:
-        config["inputs"] = "one q/k/v buffer per layer, reused by every iteration"
-    if args.profile:
-        keep = [i for i, it in enumerate(w.its) if it.chunk_size == args.profile_chunk][-2:]
-        w.its = [w.its[i] for i in keep]
-        w.descs = [w.descs[i] for i in keep]
-        w.layer_arrays = [w.layer_arrays[i] for i in keep]
-        w.work = [w.work[i] for i in keep]
-        w.tokens_per_step = sum(it.n_tokens for it in w.its)
-        config["workload"] += f"-profile-{w.L}L-p{args.profile_chunk}"
-
-    def barrier():
-        if ws > 1:
-            torch.distributed.barrier()
-
-    for _ in range(max(args.warmup, 0)):
+    for _ in range(max(warmup, 0)):
         w.run_step()
     w.ctx.sync_status()
     torch.cuda.synchronize(device)
-
     n_it = len(w.its)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_it + 1)]
-           for _ in range(args.steps)]
-    gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
-    sampler = ClockSampler(gpu_id)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(n_it + 1)] for _ in range(steps)]
     barrier()
     torch.cuda.synchronize(device)
-    sampler.start()
-    time.sleep(0.25)
+    if sampler is not None:
+        sampler.start()
+        time.sleep(0.25)
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record()
-    for s in range(args.steps):
-        w.run_step(evs[s])
+    for s_ in range(steps):
+        w.run_step(evs[s_])
     t_end.record()
     torch.cuda.synchronize(device)
-    clocks = sampler.stop()
+    clocks = sampler.stop() if sampler is not None else None
     barrier()
     w.ctx.sync_status()
     total_ms = max_over_ranks(t_start.elapsed_time(t_end), ws, device)
+    it_us = np.array([[evs[s_][i].elapsed_time(evs[s_][i + 1]) * 1e3 for i in range(n_it)]
+                      for s_ in range(steps)])
+    return total_ms, it_us, clocks
 
-    it_us = np.array([[evs[s][i].elapsed_time(evs[s][i + 1]) * 1e3 for i in range(n_it)]
-                      for s in range(args.steps)])          # [steps][iterations]
+
+def summarize(w, it_us, peaks, config_name):
+    """Per chunk size: device us P50/P99 per iteration, tokens/s, the
+    fraction of the iterations' roofline (the slower of their flops at the
+    sustained tensor peak and their bytes at the HBM peak), P99 against the
+    decode-only iteration; and the roofline object of the whole sweep."""
+    n_it = len(w.its)
     L = w.L
     hbm = peaks["hbm_gbs"] * 1e9
     tfl = peaks["bf16_tflops_sustained"] * 1e12
@@ -747,23 +726,144 @@ def main():
     if p0_p99:
         for v in per_chunk.values():
             v["p99_vs_decode_only"] = v["device_us_p99"] / p0_p99
-
     t_total = t_it.sum()
     bound = "tensor" if F.sum() / tfl > B.sum() / hbm else "hbm"
     if bound == "hbm":
         achieved, peak, unit = B.sum() / t_total / 1e9, peaks["hbm_gbs"], "GB/s"
+        peak_kind = "measured HBM copy" if peaks["source"] == "measured" else "fallback HBM"
     else:
         achieved, peak, unit = F.sum() / t_total / 1e12, peaks["bf16_tflops_sustained"], "TFLOP/s"
-    traffic = committed_traffic()
+        peak_kind = ("measured sustained bf16 GEMM" if peaks["source"] == "measured"
+                     else "fallback sustained bf16")
     roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
-                "frac": achieved / peak, "traffic": traffic,
+                "frac": achieved / peak, "traffic": committed_traffic(config_name),
                 "algorithmic_bytes_per_launch": float(B.sum() / (L * n_it)),
                 "algorithmic_flops_per_launch": float(F.sum() / (L * n_it)),
                 "avg_launch_us": float(t_total / (L * n_it) * 1e6),
                 "max_bound_frac": float(sum(max(F[i] / tfl, B[i] / hbm) for i in range(n_it))
                                         / t_total),
-                "peak_source": peaks["source"], "kernel": "mixed_layer_kernel"}
+                "peak_source": peaks["source"], "peak_kind": peak_kind,
+                "kernel": "mixed_layer_kernel"}
+    return per_chunk, roofline
 
+
+def side_config(name, steps, warmup, peaks, device, barrier):
+    """Another sweep in the same run, reported beside the headline."""
+    import torch
+    from synth import workload as wl
+    cfg = wl.CONFIGS[name]
+    w = Workload(cfg, device, lean=name in LEAN_CONFIGS)
+    total_ms, it_us, _ = time_sweep(w, steps, warmup, 1, device, barrier)
+    per_chunk, roofline = summarize(w, it_us, peaks, name)
+    out = {"value": whole_job_value(w.tokens_per_step, steps, 1, total_ms), "unit": UNIT,
+           "steps": steps, "warmup": warmup, "ms_per_step": total_ms / steps,
+           "layers": cfg.n_layers, "q_heads": cfg.hq, "decodes": cfg.n_decodes,
+           "prompt_len": cfg.prompt_len, "iterations_per_step": len(w.its),
+           "roofline": roofline, "per_chunk": per_chunk}
+    w.close()
+    del w
+    torch.cuda.empty_cache()
+    return out
+
+
+# ------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--profile", action="store_true",
+                    help="small case for ncu: 2 layers, iterations of --profile-chunk only")
+    ap.add_argument("--profile-chunk", type=int, default=2048)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-side", action="store_true", help="skip the sweeps reported beside the headline")
+    ap.add_argument("--lean", action="store_true",
+                    help="one q/k/v buffer per layer reused by all iterations (large sweeps)")
+    ap.add_argument("--workload", default="sweep", choices=["sweep", "trace"],
+                    help="trace: the completion-timed DLFP loop vs a fixed chunk cap")
+    args = ap.parse_args()
+
+    ws, rank, local = dist_setup()
+    from synth import workload as wl
+    cfg = wl.CONFIGS[args.config]
+    lean = args.lean or args.config in LEAN_CONFIGS
+    config = {"workload": cfg.name, "q_heads": cfg.hq, "kv_heads": 8, "head_dim": 128,
+              "page_size": 16, "layers": cfg.n_layers, "decodes": cfg.n_decodes,
+              "decode_ctx": f"{cfg.ctx_dist}[{cfg.ctx_lo},{cfg.ctx_hi}]",
+              "prompt_len": cfg.prompt_len, "chunk_sizes": list(cfg.chunk_sizes),
+              "iterations_per_step": len(cfg.iterations()),
+              "l2": f"inputs larger than L2: each iteration reads {cfg.n_layers} distinct "
+                    "per-layer KV pools of several hundred MB or more",
+              "parallelism": f"replicas{ws}"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        import oracle
+        fn, ntok, desc, scale = oracle_sample(cfg, "light")
+        for _ in range(args.warmup):
+            fn()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            fn()
+        dt = time.perf_counter() - t0
+        val = ntok * args.steps / (dt * scale * cfg.n_layers)
+        line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT,
+                "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": config,
+                "cpu_baseline": {"value": val, "unit": UNIT, "cores": oracle.max_threads(),
+                                 "kind": "oracle", "sample": desc},
+                "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    import torch
+    if args.workload == "trace":
+        if rank == 0:
+            device = torch.device("cuda", local)
+            torch.cuda.set_device(device)
+            res = trace_measure(device)
+            print(json.dumps({"metric": "open-loop trace: per-iteration device us P50/P99 and "
+                              "ITL/TTFT, completion-timed DLFP vs fixed chunk caps",
+                              "workload": "qwen3-0.6b-attn-28L-poisson-trace", **res}))
+        return
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    peaks = load_peaks()
+
+    layers = 2 if args.profile else None
+    w = Workload(cfg, device, seed_offset=replica_seed_offset(rank), layers=layers, lean=lean)
+    if lean:
+        config["inputs"] = "one q/k/v buffer per layer, reused by every iteration"
+    if args.profile:
+        keep = [i for i, it in enumerate(w.its) if it.chunk_size == args.profile_chunk][-2:]
+        w.its = [w.its[i] for i in keep]
+        w.descs = [w.descs[i] for i in keep]
+        w.layer_arrays = [w.layer_arrays[i] for i in keep]
+        w.work = [w.work[i] for i in keep]
+        w.inputs = [w.inputs[i] for i in keep]
+        w.tokens_per_step = sum(it.n_tokens for it in w.its)
+        config["workload"] += f"-profile-{w.L}L-p{args.profile_chunk}"
+
+    def barrier():
+        if ws > 1:
+            torch.distributed.barrier()
+
+    gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
+    total_ms, it_us, clocks = time_sweep(w, args.steps, args.warmup, ws, device, barrier,
+                                         ClockSampler(gpu_id))
+    per_chunk, roofline = summarize(w, it_us, peaks, args.config if not args.profile else None)
+    n_it = len(w.its)
     value = whole_job_value(w.tokens_per_step, args.steps, ws, total_ms)
     plan = w.ctx.last_plan()
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
@@ -772,16 +872,26 @@ def main():
             "data": "synthetic (seeded N(0,1) bf16, random page permutation)",
             "config": config, "roofline": roofline, "per_chunk": per_chunk,
             # per iteration: one plan-upload kernel and one mixed_layer_kernel per layer
-            "gpu_launches": (L + 1) * n_it * args.steps, "clocks": clocks,
+            "gpu_launches": (w.L + 1) * n_it * args.steps, "clocks": clocks,
             "plan_last": plan}
     if not args.no_e2e and not args.profile:
         line["e2e"] = e2e_measure(w, max(1, min(args.steps, 3)), device)
     if not args.profile:
-        line["independent_layers"] = independent_layers_measure(w, args.steps, ws, device)
-    if not args.profile and args.config == "qwen3-0.6b-attn-28L-chunk-sweep" and rank == 0:
-        line["several_chunks"] = several_chunks_measure(cfg, peaks, device)
+        line["independent_layers"] = independent_layers_measure(w, max(1, min(args.steps, 3)), ws, device)
     if rank == 0 and ws == 1 and not args.no_cpu and not args.profile:
         line["cpu_baseline"] = cpu_baseline(cfg)
+    w.close()
+    del w
+    torch.cuda.empty_cache()
+    if not args.profile and not args.no_side and ws == 1:
+        side = {}
+        for name in SIDE_CONFIGS:
+            if name != args.config:
+                side[name] = side_config(name, max(1, min(args.steps, 5)), 2, peaks, device, barrier)
+        line["other_configs"] = side
+        if "qwen3-0.6b-attn-28L-chunk-sweep" in wl.CONFIGS:
+            line["several_chunks"] = several_chunks_measure(wl.CONFIGS["qwen3-0.6b-attn-28L-chunk-sweep"],
+                                                            peaks, device)
     if rank == 0:
         print(json.dumps(line))
     if ws > 1:
