@@ -161,9 +161,12 @@ int mx_mixed_attention(mx_ctx *ctx, const mx_iter_desc *desc,
                        const mx_layer_bufs *bufs, void *stream);
 
 /* A whole iteration: the same schedule `desc` run through n_layers layers
- * (layers[l] holds layer l's tensors), one launch per layer, planned once.
- * The layers' tensors must be distinct (no layer reads what another writes):
- * consecutive layer launches may overlap on the GPU (see MX_OPT_PDL).
+ * (layers[l] holds layer l's tensors), one launch per layer, planned once,
+ * in order: with MX_OPT_PDL 0 or 1 (the default), layer l+1 reads its
+ * tensors only after layer l has completed, so layer l+1's q/k/v may be what
+ * layer l wrote (its out, or data derived from it in place).  With
+ * MX_OPT_PDL 2 consecutive layers overlap on the GPU and must be independent
+ * (distinct tensors; no layer reads what another writes).
  * With device_us_out != NULL: records CUDA events before the first and after
  * the last launch, waits for the second, and stores the elapsed device time in
  * microseconds in *device_us_out (the L_t of Eq. 1 as completed on the
@@ -179,7 +182,9 @@ int mx_iteration(mx_ctx *ctx, const mx_iter_desc *desc, int32_t n_layers,
 int mx_sync_status(mx_ctx *ctx, void *stream);
 
 /* Copy a NUL-terminated description of the context's last failure into buf
- * (at most len bytes).  Returns the length written, or MX_EINVAL. */
+ * (at most len bytes).  With ctx == NULL: why the calling thread's last
+ * mx_create failed (empty after a successful one).  Returns the length
+ * written, or MX_EINVAL (buf NULL or len <= 0). */
 int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
 
 /* Tunables.  MX_OPT_SPLIT_KEYS: keys per decode split (multiple of 128,
@@ -191,8 +196,9 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
 #define MX_OPT_GRID 2
 #define MX_OPT_PREFILL_PIECE_TILES 3
 /* MX_OPT_PDL: how the layer launches of mx_iteration follow each other.
- * 1 (default): programmatic dependent launch hides the launch latency, and
- * layer l+1 starts working once layer l has finished: the order of a model
+ * 1 (default): programmatic dependent launch hides the launch latency; each
+ * CTA of layer l+1 waits (griddepcontrol.wait) until layer l has completed
+ * and its writes are visible before it reads anything: the order of a model
  * whose layer l+1 attention reads what layer l produced.  2: the layers are
  * independent problems; layer l+1's CTAs start on the SMs layer l frees,
  * filling layer l's tail (needs a grid of every SM, else behaves as 1).
@@ -220,9 +226,10 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  * schedulers and tests can inspect it).  The paper schedules per iteration a
  * decode set D_t and a prefill chunk of p_t tokens (§2.1, Eq. 1); one launch
  * splits that work into items that its persistent CTAs claim in order:
- * prefill query tiles (128 rows x one query head, or a key piece of one),
- * heaviest first, then decode splits (one decode x one KV head x a key
- * range), longest first.
+ * prefill query tiles (128 rows x two query heads of one KV head, or one
+ * head when num_q_heads == num_kv_heads; or a key piece of one), heaviest
+ * first, then decode splits (one decode x one KV head x a key range),
+ * longest first.
  *
  * geom and desc as for mx_create / mx_mixed_attention (desc's page_table and
  * slots are not read and may be NULL); num_sms: the SM count the launch will
@@ -230,11 +237,14 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  * MX_OPT_PREFILL_PIECE_TILES and MX_OPT_PDL (0, 0 and 1 are the defaults).
  * Outputs (host arrays owned by the caller):
  *   items    int32 [max_items][4], n_items records in claim order:
- *     prefill {f << 4, t | hq << 16, s | n_s << 16, partial slot base}:
- *       piece s of n_s of query tile t (rows [128 t, 128 t + 128) of prefill
- *       chunk f, in the order of desc->prefills, or 0 for the single chunk)
- *       of query head hq; the tile's n_T = ceil(chunk_start_f / 128) + t + 1
- *       key tiles (128 keys each) are split as [s n_T / n_s, (s + 1) n_T / n_s);
+ *     prefill {f << 4 | (heads - 1) << 8, t | hq << 16, s | n_s << 16,
+ *       partial slot base}: piece s of n_s of query tile t (rows
+ *       [128 t, 128 t + 128) of prefill chunk f, in the order of
+ *       desc->prefills, or 0 for the single chunk) of query heads hq ..
+ *       hq + heads - 1 (heads 1 or 2); the tile's n_T =
+ *       ceil(chunk_start_f / 128) + t + 1 key tiles (128 keys each) are split
+ *       as [s n_T / n_s, (s + 1) n_T / n_s); head e of piece s writes partial
+ *       slot base + e n_s + s when n_s > 1;
  *     decode {1 | h << 4 | s << 11 | (len / 16) << 23, decode index i,
  *       page-table row, cached tokens ctx}: split s of decode i, KV head h,
  *       keys [s len, min((s + 1) len, ctx + 1)); kind 2 instead of 1 for a

@@ -165,7 +165,9 @@ class Context:
         h = ctypes.c_void_p()
         rc = self._lib.mx_create(ctypes.byref(h), ctypes.byref(self.geom), device)
         if rc != MX_OK:
-            raise MxError(rc, "mx_create failed")
+            buf = ctypes.create_string_buffer(512)
+            self._lib.mx_error_detail(None, buf, 512)
+            raise MxError(rc, "mx_create: " + buf.value.decode(errors="replace"))
         self._h = h
 
     def close(self):

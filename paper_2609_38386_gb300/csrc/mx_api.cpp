@@ -96,6 +96,21 @@ struct mx_ctx {
 
 namespace {
 
+// Why the calling thread's last mx_create failed (there is no context to
+// hold it); mx_error_detail(NULL, ...) returns it.
+thread_local std::string t_create_error;
+
+int create_fail(int code, const char *fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    t_create_error = buf;
+    return code;
+}
+
 int fail(mx_ctx *c, int code, const char *fmt, ...)
 {
     if (c) {
@@ -342,21 +357,25 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
     if (count_parts(split) > kPartSlots)
         return fail_to(err, MX_ECAPACITY, "decode splits exceed the partial workspace");
 
-    // Prefill tiles, split along their key tiles into pieces of at most
-    // piece_tiles tiles so that long causal rows spread over several SMs.
+    // Prefill items: a query tile of two query heads of one KV head (one K/V
+    // tile load serves both; one head when Hq = Hkv), split along their key
+    // tiles into pieces of at most piece_tiles tiles so that long causal rows
+    // spread over several SMs.
+    const int nh = hq / hkv >= 2 ? 2 : 1;   // heads per prefill item
+    const int n_grp = hq / nh;              // prefill items per query tile
     int n = 0;
     int64_t pre_work = 0;
     for (const PrefillInfo &x : pfs) {
         const int nA = (x.chunk_start + kTileN - 1) / kTileN;
         for (int t = 0; t < (x.p_t + kTileM - 1) / kTileM; ++t)
-            pre_work += (int64_t)(nA + t + 1) * hq;
+            pre_work += (int64_t)(nA + t + 1) * n_grp;
     }
     // Splitting costs a partial write and a merge; it pays only when the
     // chunk has too few tiles to occupy the GPU (short chunks deep into a
     // long prompt), so tiles are split only then, into >= 48-tile pieces.
     int piece = k.piece_tiles_opt;
     if (piece <= 0) {
-        if ((int64_t)n_qt * hq * 2 >= k.num_sms)
+        if ((int64_t)n_qt * n_grp * 2 >= k.num_sms)
             piece = 65535;
         else
             piece = (int)std::max<int64_t>(kMinPieceTiles, (pre_work + k.num_sms - 1) / k.num_sms);
@@ -368,7 +387,7 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
             for (int t = 0; t < (x.p_t + kTileM - 1) / kTileM; ++t) {
                 const int ns = (nA + t + 1 + pc - 1) / pc;
                 if (ns > 1)
-                    parts += (int64_t)ns * hq;
+                    parts += (int64_t)ns * hq;   // one partial per piece and head
             }
         }
         return parts;
@@ -385,13 +404,13 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
         for (int t = (pfs[f].p_t + kTileM - 1) / kTileM - 1; t >= 0; --t) {
             const int nT = nA + t + 1;
             const int ns = (nT + piece - 1) / piece;
-            for (int h = 0; h < hq; ++h) {
+            for (int gq = 0; gq < n_grp; ++gq) {
                 const int base = ns > 1 ? pre_part : 0;
                 if (ns > 1)
-                    pre_part += ns;
+                    pre_part += ns * nh;   // head e of piece s: base + e * ns + s
                 for (int s2 = 0; s2 < ns; ++s2) {
                     const int len = (int)((int64_t)(s2 + 1) * nT / ns - (int64_t)s2 * nT / ns);
-                    pitems.push_back({len, prefill_item_code(f, t, h, s2, ns, base)});
+                    pitems.push_back({len, prefill_item_code(f, t, gq * nh, nh, s2, ns, base)});
                 }
             }
         }
@@ -658,18 +677,22 @@ extern "C" {
 
 int mx_create(mx_ctx **out, const mx_geom *g, int device)
 {
+    t_create_error.clear();
     if (!out || !g)
-        return MX_EINVAL;
+        return create_fail(MX_EINVAL, "null out or geometry");
     *out = nullptr;
     if (!geom_ok(*g))
-        return MX_EINVAL;
+        return create_fail(MX_EINVAL,
+                           "unsupported geometry: head_dim must be 128, page_size 16, Hq / Hkv a power of "
+                           "two of at most 8, Hkv <= %d, and the sizes positive",
+                           kMaxDecodeKvHeads);
     int ndev = 0;
     if (cudaGetDeviceCount(&ndev) != cudaSuccess || device < 0 || device >= ndev)
-        return MX_EDEVICE;
+        return create_fail(MX_EDEVICE, "device %d: no such CUDA device (%d found)", device, ndev);
     DeviceGuard guard(device);
     cudaDeviceProp prop;
     if (cudaGetDeviceProperties(&prop, device) != cudaSuccess || prop.major != 10)
-        return MX_EDEVICE;
+        return create_fail(MX_EDEVICE, "device %d is not an sm_100-family GPU", device);
 
     mx_ctx *c = new mx_ctx();
     c->g = *g;
@@ -681,10 +704,8 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     c->max_items = max_prefill_items + kPartSlots + std::max(g->max_decodes, 1) * g->num_kv_heads;
 
     auto bail = [&](cudaError_t e, const char *what) {
-        std::string msg = std::string(what) + ": " + cudaGetErrorString(e);
         mx_destroy(c);
-        (void)msg;
-        return MX_ECUDA;
+        return create_fail(MX_ECUDA, "%s: %s", what, cudaGetErrorString(e));
     };
     cudaError_t e;
     if ((e = init_layer_kernel()) != cudaSuccess)
@@ -756,7 +777,7 @@ int mx_create(mx_ctx **out, const mx_geom *g, int device)
     e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
     if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) {
         mx_destroy(c);
-        return MX_ECUDA;
+        return create_fail(MX_ECUDA, "cuTensorMapEncodeTiled entry point not found");
     }
     c->encode = reinterpret_cast<EncodeTiledFn>(fn);
     if ((e = cudaDeviceSynchronize()) != cudaSuccess)
@@ -867,17 +888,19 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     cudaError_t e;
     if (timed && (e = cudaEventRecord(c->ev_start, st)) != cudaSuccess)
         return cuda_fail(c, e, "cudaEventRecord(start)");
-    // Layers of one iteration are independent (distinct tensors), so layer
-    // l > 0 may start while layer l - 1 drains; the first layer keeps
-    // ordinary stream order behind whatever the caller enqueued before.
+    // Layer l > 0 is launched with programmatic dependent launch; the first
+    // layer keeps ordinary stream order behind whatever the caller enqueued
+    // before.
     for (int l = 0; work && l < n_layers; ++l) {
-        // Mode 1: layer l+1 launches as layer l's CTAs run out of work and
-        // starts once layer l has completed (launch latency hidden, no
-        // overlap: the order a model whose layers depend on each other
-        // imposes).  Mode 2: layer l+1's CTAs start on the SMs layer l frees.
-        // That is safe only when a launch occupies every SM (one CTA per SM):
-        // then launch n + 3 cannot start before launch n has completed (see
-        // kWorkSets); smaller grids keep mode 1.
+        // Mode 1: layer l+1 launches as layer l's CTAs run out of work, and
+        // each of its CTAs waits for layer l to complete (griddepcontrol.wait)
+        // before reading anything: layer l+1 may read what layer l wrote, the
+        // order of a model whose layers depend on each other, with the launch
+        // latency hidden.  Mode 2 (independent layers only): layer l+1's CTAs
+        // start on the SMs layer l frees.  That is safe only when a launch
+        // occupies every SM (one CTA per SM): then launch n + 3 cannot start
+        // before launch n has completed (see kWorkSets); smaller grids keep
+        // mode 1.
         const int grid = grid_for(c, pl);
         params[l].early_start = (c->pdl == 2 && grid == c->num_sms) ? 1 : 0;
         e = launch_mixed_layer(params[l], grid, st, c->pdl != 0 && l > 0);
@@ -913,10 +936,11 @@ int mx_sync_status(mx_ctx *c, void *stream)
 
 int mx_error_detail(mx_ctx *c, char *buf, int32_t len)
 {
-    if (!c || !buf || len <= 0)
+    if (!buf || len <= 0)
         return MX_EINVAL;
-    const size_t n = std::min<size_t>(c->last_error.size(), (size_t)len - 1);
-    std::memcpy(buf, c->last_error.data(), n);
+    const std::string &msg = c ? c->last_error : t_create_error;
+    const size_t n = std::min<size_t>(msg.size(), (size_t)len - 1);
+    std::memcpy(buf, msg.data(), n);
     buf[n] = '\0';
     return (int)n;
 }

@@ -10,9 +10,21 @@ namespace mx {
 
 constexpr int kHeadDim = 128;
 constexpr int kPage = 16;
-constexpr int kThreads = 256;            // 8 warps per CTA
-constexpr int kWarps = kThreads / 32;
+// 12 warps per CTA: warpgroup 0 (warps 0-3) loads tiles and issues the
+// tensor-core MMAs of prefill items; warpgroups 1 and 2 (the 256 "consumer"
+// threads) run the softmax of one query head each in prefill items and all
+// of a decode item.
+constexpr int kThreads = 384;
+constexpr int kProdThreads = 128;
+constexpr int kConsThreads = kThreads - kProdThreads;   // 256
+constexpr int kWarps = kConsThreads / 32;               // warps of a decode item (8)
 constexpr int kMaxRep = 8;               // Hq / Hkv supported up to 8
+// Registers per thread after the split (setmaxnreg): the launch gives 168
+// to each of the 384 threads (64512); warpgroup 0 keeps 56, the consumers
+// take 224: 128 x 56 + 256 x 224 = 64512.
+constexpr int kProdRegs = 56;
+constexpr int kConsRegs = 224;
+static_assert(kProdThreads * kProdRegs + kConsThreads * kConsRegs <= kThreads * 168, "register split");
 
 // Prefill tile geometry: 128 query rows x 128 keys per tcgen05 tile.
 constexpr int kTileM = 128;
@@ -21,32 +33,35 @@ constexpr int kTileN = 128;
 // Shared-memory plan (bytes, offsets from a 1024-aligned base).
 constexpr int kHalfTile = kTileM * 64 * 2;             // 128 rows x 64 bf16 = 16 KiB
 constexpr int kTileBytes = 2 * kHalfTile;              // 32 KiB
-// K stage c % 3 is released by the completion of S_c = Q K_c^T (the same
-// barrier that hands S_c to the softmax) and V stage c % 2 by that of P_c V_c;
-// the loads run two to three tiles ahead of their use.
-constexpr int kKStages = 3;
+// A prefill item serves one or two query heads of one KV head: a Q tile per
+// head, and K / V rings shared by both.  K stage c % kKStages is released
+// once both heads' S_c = Q K_c^T have completed, V stage c % kVStages once
+// both heads' P_c V_c have.
+constexpr int kKStages = 2;
 constexpr int kVStages = 2;
-constexpr int kSmemQ = 0;
-constexpr int kSmemK = kSmemQ + kTileBytes;
+constexpr int kSmemQ = 0;                              // Q of head 0, then head 1
+constexpr int kSmemK = kSmemQ + 2 * kTileBytes;
 constexpr int kSmemV = kSmemK + kKStages * kTileBytes;
 constexpr int kSmemData = kSmemV + kVStages * kTileBytes;   // 192 KiB
 constexpr int kSmemMisc = kSmemData;                   // barriers etc.
 constexpr int kSmemMiscBytes = 1024;
 constexpr int kSmemTotal = kSmemData + kSmemMiscBytes + 1024;  // + alignment slack
 
-// Decode ring: each warp owns kDecStages stages of one page (K 4 KiB + V 4 KiB).
+// Decode ring: each of the 8 decode warps owns kDecStages stages of one page
+// (K 4 KiB + V 4 KiB).
 constexpr int kPageBytes = kPage * kHeadDim * 2;       // 4 KiB
 constexpr int kDecStageBytes = 2 * kPageBytes;         // 8 KiB
 constexpr int kDecStages = 3;
 static_assert(kWarps * kDecStages * kDecStageBytes <= kSmemData, "decode ring too large");
 
-// TMEM columns: three S buffers [0,128), [128,256), [256,384) (fp32) and O
-// [384,512) (fp32).  P_b (bf16 pairs, the A operand of P.V) overwrites the
-// first 64 columns of S_b once they are read.  Three S buffers let Q.K^T run
-// two key tiles ahead of P.V, so the softmax never waits for its scores.
+// TMEM columns (fp32): S of head 0 [0,128), S of head 1 [128,256), O of
+// head 0 [256,384), O of head 1 [384,512).  P_h (bf16 pairs, the A operand
+// of P.V) overwrites the first 64 columns of S_h once they are read; the next
+// S_h = Q K^T is issued after that P.V, so the tensor pipe's in-order
+// execution keeps the two apart.
 constexpr uint32_t kTmemCols = 512;
-constexpr int kSBuf = 3;
-constexpr uint32_t kTmemO = kSBuf * 128;
+constexpr uint32_t kTmemS = 0;
+constexpr uint32_t kTmemO = 256;
 
 enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1, ITEM_DECODE_SHORT = 2 };
 
@@ -62,10 +77,12 @@ struct PrefillInfo {
 };
 
 // Work-item encodings (int4):
-//   prefill: {ITEM_PREFILL | chunk f << 4, t | hq << 16, s | n_s << 16,
-//             partial slot base}: piece s of n_s of query tile t (rows
-//            [128t, 128t+128) of chunk f) of head hq; the tile's key tiles are
-//            split evenly between its n_s pieces.
+//   prefill: {ITEM_PREFILL | chunk f << 4 | (heads - 1) << 8, t | hq << 16,
+//             s | n_s << 16, partial slot base}: piece s of n_s of query tile
+//            t (rows [128t, 128t+128) of chunk f) of query heads hq .. hq +
+//            heads - 1 (heads 1 or 2, one KV head); the tile's key tiles are
+//            split evenly between its n_s pieces; head e of piece s writes
+//            partial slot base + e * n_s + s.
 //   short decode (at most 16 keys, one split): the decode record with kind
 //            ITEM_DECODE_SHORT;
 //   decode:  {ITEM_DECODE | kv head << 4 | split index << 11 | split
@@ -73,10 +90,10 @@ struct PrefillInfo {
 //             split s of decode i covers keys [s * len, (s + 1) * len) of
 //             [0, ctx]; the row, length and split size travel in the item so
 //             that the page-id loads need no other lookup first
-__host__ __device__ inline int4 prefill_item_code(int f, int t, int hq, int s, int n_s, int part_base)
+__host__ __device__ inline int4 prefill_item_code(int f, int t, int hq, int heads, int s, int n_s, int part_base)
 {
     int4 r;
-    r.x = ITEM_PREFILL | (f << 4);
+    r.x = ITEM_PREFILL | (f << 4) | ((heads - 1) << 8);
     r.y = t | (hq << 16);
     r.z = s | (n_s << 16);
     r.w = part_base;

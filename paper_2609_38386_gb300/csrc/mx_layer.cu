@@ -7,19 +7,30 @@
 // 1/sqrt(128); a decode with ctx cached tokens sees ctx + 1 keys; chunk row j
 // sees keys [0, chunk_start + j].
 //
+// CTA: 12 warps.  Warpgroup 0 (warps 0-3, few registers) loads tiles and
+// issues tensor-core MMAs; warpgroups 1 and 2 (the 256 "consumer" threads,
+// many registers) run the softmax and epilogue of prefill items and the whole
+// of decode items.  Each role runs its own copy of the persistent item loop;
+// the roles meet at a named barrier between items.
+//
 // Work items (built on the host, fetched with one atomic counter):
-//   ITEM_PREFILL {t, hq, piece}: 128 chunk rows [128t, 128t+128) of query
-//                           head hq against one contiguous range of its key
-//                           tiles, on tcgen05 tensor cores (S and O
-//                           accumulators in TMEM).  A tile with several pieces
-//                           writes (O, lse) partials; the last-arriving piece
-//                           merges them.  Piece 0 of each of the n_rep
-//                           query heads of a KV head appends 128 / n_rep of
-//                           the tile's tokens to the KV cache.
-//   ITEM_DECODE  {h, s | i | seq | ctx}: split s of decode i's keys for KV head h, all n_rep
-//                           query heads of the group at once: a split-KV
-//                           flash-decode whose partial (O, lse) is merged by
-//                           the last-arriving split (no waiting).
+//   ITEM_PREFILL {t, hq, heads, piece}: 128 chunk rows [128t, 128t+128) of
+//                           query heads hq (and hq + 1 when heads = 2, the
+//                           same KV head) against one contiguous range of
+//                           their key tiles, on tcgen05 tensor cores (S and O
+//                           accumulators of both heads in TMEM, one K/V tile
+//                           load for both).  Warp 0 loads Q and K, warp 2 V,
+//                           warp 1 issues the MMAs; consumer warpgroup e runs
+//                           the softmax of head hq + e.  A tile with several
+//                           pieces writes (O, lse) partials; the last-arriving
+//                           piece merges them.  Piece 0 of each of the
+//                           n_rep / heads items of a KV head appends its share
+//                           of the tile's tokens to the KV cache.
+//   ITEM_DECODE  {h, s | i | seq | ctx}: split s of decode i's keys for KV
+//                           head h, all n_rep query heads of the group at
+//                           once: a split-KV flash-decode whose partial
+//                           (O, lse) is merged by the last-arriving split (no
+//                           waiting).
 //   ITEM_DECODE_SHORT: a decode of at most 16 keys, exact on CUDA cores.
 // New keys/values are read from the k/v inputs, never from the pages being
 // written in the same launch, so the append needs no ordering.
@@ -32,23 +43,27 @@
 namespace mx {
 
 struct Misc {
-    uint64_t bar_q;
-    uint64_t bar_kfull[kKStages];
-    uint64_t bar_sfull[kSBuf];
-    // P_c written (128 softmax arrivals) and V tile c landed (the V
-    // producer's arrive + transaction bytes): the one wait before P_c V_c
-    uint64_t bar_pfull[kSBuf];
-    uint64_t bar_odone[2];  // P_c V_c done (c & 1); frees V stage c % 2
-    uint64_t bar_never;     // fault injection: a barrier nothing arrives at
+    uint64_t bar_q;                   // Q tiles of the item landed
+    uint64_t bar_kfull[kKStages];     // K tile landed
+    uint64_t bar_kempty[kKStages];    // both heads' S = Q K^T of that tile done
+    uint64_t bar_vfull[kVStages];     // V tile landed
+    uint64_t bar_vempty[kVStages];    // both heads' P V of that tile done
+    uint64_t bar_sfull[2];            // S_h ready for head h's softmax
+    uint64_t bar_pfull[2];            // P_h written by head h's 128 softmax threads
+    uint64_t bar_odone;               // every MMA of the item done
+    uint64_t bar_never;               // fault injection: a barrier nothing arrives at
     uint32_t tmem_base;
     int32_t item_idx[2];
     int32_t abort;
     int32_t last;
-    PrefillInfo pre[kMaxPrefills];  // the launch's prefill chunks
+    PrefillInfo pre[kMaxPrefills];    // the launch's prefill chunks
 };
 static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
-static_assert(kVStages == 2, "V stage c % 2 is released by the odone barrier c & 1");
-static_assert(kKStages == kSBuf, "K stage c % 3 is released by the sfull barrier c % 3");
+
+// Named barriers: 1 = every thread of the CTA between items, 2 = the 256
+// consumer threads (0 is __syncthreads, used only outside the item loops).
+constexpr uint32_t kBarItem = 1, kBarCons = 2;
+__device__ __forceinline__ void cons_sync() { named_sync(kBarCons, kConsThreads); }
 
 // Instruction descriptors: S = Q K^T (both K-major) and O = P V (V MN-major).
 constexpr uint32_t kIdescS = idesc_bf16_f32(128, 128, false, false);
@@ -75,9 +90,9 @@ __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000);
 // scores go through shared memory; cached K/V rows are read from their page,
 // the new key from the k/v inputs (as in the split path), which it appends.
 // ---------------------------------------------------------------------------
-__device__ void decode_short_item(const LayerParams &P, uint8_t *smem, int di, int h, int seq, int n)
+__device__ void decode_short_item(const LayerParams &P, uint8_t *smem, int di, int h, int seq, int n, int tid)
 {
-    const int tid = threadIdx.x, nrep = P.n_rep, nk = n + 1;
+    const int nrep = P.n_rep, nk = n + 1;   // tid: consumer thread 0..255
     float *ss = reinterpret_cast<float *>(smem);  // [kMaxRep][16] scores (log2 domain)
     if (tid < 32) {
         const int slot = P.slots[di];
@@ -125,8 +140,8 @@ __device__ void decode_short_item(const LayerParams &P, uint8_t *smem, int di, i
         }
         ss[q * kPage + k] = s;
     }
-    __syncthreads();
-    for (int e = tid; e < nrep * kHeadDim; e += kThreads) {
+    cons_sync();
+    for (int e = tid; e < nrep * kHeadDim; e += kConsThreads) {
         const int q = e / kHeadDim, d = e % kHeadDim;
         float m = neg_inf();
         for (int k = 0; k < nk; ++k)
@@ -195,9 +210,10 @@ __device__ __forceinline__ void decode_issue_page(const LayerParams &P, uint32_t
 }
 
 __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int di, int h,
-                            int s, int seq, int n, int split_len)
+                            int s, int seq, int n, int split_len, int tid)
 {
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // tid: consumer thread 0..255, warp: decode warp 0..7
+    const int warp = tid >> 5, lane = tid & 31;
     // split count and partial slots are needed only at the end: the load
     // overlaps the page-id loads (the row and length came with the item)
     const DecodeInfo D = P.dec[di];
@@ -349,17 +365,10 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
         l0 += p0 + p2;
         l1 += p1 + p3;
         // P^T as the B operand (keys x query rows): transpose the 8x8 blocks
-        const uint32_t h01 = pack_bf16(p0, p1), h23 = pack_bf16(p2, p3);
-        const uint32_t b0 = movmatrix_t(h01);
-        const uint32_t b1 = movmatrix_t(h23);
-        // A decode of at most 16 keys takes P as hi + lo (p minus its bf16
-        // rounding): with so few keys one weight's rounding shows in O.
-        const bool lo = n < kPage;
-        uint32_t c0 = 0u, c1 = 0u;
-        if (lo) {
-            c0 = movmatrix_t(pack_bf16(p0 - bf16lo(h01), p1 - bf16hi(h01)));
-            c1 = movmatrix_t(pack_bf16(p2 - bf16lo(h23), p3 - bf16hi(h23)));
-        }
+        // (decodes of at most 16 keys, where the bf16 rounding of one weight
+        // would show, are ITEM_DECODE_SHORT items and never come here)
+        const uint32_t b0 = movmatrix_t(pack_bf16(p0, p1));
+        const uint32_t b1 = movmatrix_t(pack_bf16(p2, p3));
         // O^T (128 d x 8 rows) += V^T (128 x 16 keys) * P^T (16 x 8)
         {
             const int mi = lane >> 3;
@@ -370,7 +379,6 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
                 uint32_t a0, a1, a2, a3;
                 ldsm_x4_t(vbase + key * 256 + ((chunk ^ (key & 7)) << 4), a0, a1, a2, a3);
                 mma_bf16_16816(acc[mt], a0, a1, a2, a3, b0, b1);
-
             }
         }
         __syncwarp();
@@ -383,8 +391,8 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
         l1 += __shfl_xor_sync(0xffffffffu, l1, o);
     }
 
-    // ---- combine the 8 warps of the CTA (shared memory)
-    __syncthreads();
+    // ---- combine the 8 decode warps (shared memory)
+    cons_sync();
     float *so = reinterpret_cast<float *>(smem);               // [warp][8][128]
     float *sml = so + kWarps * kMaxRep * kHeadDim;              // [warp][8][2]
 #pragma unroll
@@ -401,11 +409,11 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
         sml[(warp * kMaxRep + 2 * tq + 1) * 2 + 0] = m1;
         sml[(warp * kMaxRep + 2 * tq + 1) * 2 + 1] = l1;
     }
-    __syncthreads();
+    cons_sync();
 
     const int nsp = D.n_splits;
     const int pslot = D.part_base + h * nsp + s;
-    for (int e = tid; e < nrep * kHeadDim; e += kThreads) {
+    for (int e = tid; e < nrep * kHeadDim; e += kConsThreads) {
         const int q = e / kHeadDim, d = e % kHeadDim;
         float M = neg_inf();
 #pragma unroll
@@ -437,17 +445,17 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
 
     // ---- cross-split merge by the last-arriving split (no waiting)
     __threadfence();
-    __syncthreads();
+    cons_sync();
     if (tid == 0) {
         const uint32_t prev = atomicAdd(P.merge_cnt + di * P.hkv + h, 1u);
         misc->last = (prev == (uint32_t)(nsp - 1)) ? 1 : 0;
     }
-    __syncthreads();
+    cons_sync();
     if (!misc->last)
         return;
     __threadfence();
     const int base = D.part_base + h * nsp;
-    for (int e = tid; e < nrep * kHeadDim; e += kThreads) {
+    for (int e = tid; e < nrep * kHeadDim; e += kConsThreads) {
         const int q = e / kHeadDim, d = e % kHeadDim;
         float M = neg_inf();
         for (int sp = 0; sp < nsp; ++sp)
@@ -501,12 +509,7 @@ __device__ __forceinline__ float row_max(const uint32_t (&sv)[128])
 
 // p = 2^(s*scale - m) of one S row as bf16 pairs into TMEM at taddr (64
 // columns), and the row sum of p in 4 packed pair chains.
-// With lo set, the low-order part of P (p minus its bf16 rounding) goes to
-// the second half of S_c as well: rows with only a few keys (the first rows
-// of a prompt) would show the rounding of a single weight of P in the
-// output, so their P.V takes P as hi + lo.
-__device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float sl, float nm, uint32_t taddr,
-                                               bool lo)
+__device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float sl, float nm, uint32_t taddr)
 {
     float rs8[8];
 #pragma unroll
@@ -525,17 +528,6 @@ __device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float 
             pk[cc] = pack_bf16(e0, e1);
         }
         tmem_st32(taddr + 32 * half, pk);
-        if (lo) {
-#pragma unroll
-            for (int cc = 0; cc < 32; ++cc) {
-                const int k0 = 64 * half + 2 * cc;
-                float x0, x1;
-                ffma2(x0, x1, __uint_as_float(sv[k0]), __uint_as_float(sv[k0 + 1]), sl, sl, nm, nm);
-                const float e0 = ex2(x0), e1 = ex2(x1);
-                pk[cc] = pack_bf16(e0 - bf16lo(pk[cc]), e1 - bf16hi(pk[cc]));
-            }
-            tmem_st32(taddr + 64 + 32 * half, pk);
-        }
     }
     return ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
 }
@@ -550,14 +542,16 @@ __device__ __forceinline__ uint4 sw128_chunk(uint32_t base, int row, int c)
     return v;
 }
 
-// Chunk row r < 16 of a chunk that starts at position 0 attends only keys
-// 0..r.  With so few keys the bf16 rounding of a single weight of P would
-// show in the output, so such a row is recomputed here in fp32 from the Q,
-// K and V tiles still in shared memory (the item's only key tile) and its
-// output row overwritten.
-__device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKt, uint32_t sVt, int r, float sl,
-                                                uint16_t *orow)
+// Chunk row r of a chunk that starts at position cs, with cs + r < 16,
+// attends only keys 0..cs+r.  With so few keys the bf16 rounding of a single
+// weight of P would show in the output, so such a row is recomputed here in
+// fp32 from the tiles still in shared memory and its output row overwritten:
+// key k < cs is row k of the cached tile (sKa, sVa: the item's first key
+// tile), key k >= cs is row k - cs of the chunk's own first tile (sKb, sVb).
+__device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKa, uint32_t sVa, uint32_t sKb,
+                                                uint32_t sVb, int cs, int r, float sl, uint16_t *orow)
 {
+    const int last = cs + r;   // keys 0..last, last < 16
     float s[16];
 #pragma unroll
     for (int k = 0; k < 16; ++k)
@@ -568,8 +562,8 @@ __device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKt, uint3
         const uint32_t qw[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
-            if (k <= r) {
-                const uint4 k4 = sw128_chunk(sKt, k, c);
+            if (k <= last) {
+                const uint4 k4 = k < cs ? sw128_chunk(sKa, k, c) : sw128_chunk(sKb, k - cs, c);
                 const uint32_t kw[4] = {k4.x, k4.y, k4.z, k4.w};
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
@@ -580,12 +574,12 @@ __device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKt, uint3
     float m = neg_inf();
 #pragma unroll
     for (int k = 0; k < 16; ++k)
-        if (k <= r)
+        if (k <= last)
             m = fmaxf(m, s[k] * sl);
     float l = 0.f;
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
-        s[k] = k <= r ? ex2(s[k] * sl - m) : 0.f;
+        s[k] = k <= last ? ex2(s[k] * sl - m) : 0.f;
         l += s[k];
     }
     const float inv = 1.0f / l;
@@ -597,8 +591,8 @@ __device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKt, uint3
             acc[e] = 0.f;
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
-            if (k <= r) {
-                const uint4 v4 = sw128_chunk(sVt, k, c);
+            if (k <= last) {
+                const uint4 v4 = k < cs ? sw128_chunk(sVa, k, c) : sw128_chunk(sVb, k - cs, c);
                 const uint32_t vw[4] = {v4.x, v4.y, v4.z, v4.w};
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
@@ -617,404 +611,558 @@ __device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKt, uint3
 }
 
 // ---------------------------------------------------------------------------
-// Prefill tile: rows [128t, 128t + 128) of the chunk, query head hq.
-// Key tiles: nA paged tiles covering [0, chunk_start), then t + 1 tiles of
-// the chunk's own keys read from the k/v inputs.
+// Prefill item: rows [128t, 128t + 128) of the chunk, query heads hq0 ..
+// hq0 + nh - 1 (one KV head), key tiles kt0 .. kt1 - 1 of the tile's nA + t + 1
+// (nA paged tiles covering [0, chunk_start), then t + 1 tiles of the chunk's
+// own keys read from the k/v inputs).  Counters carried across items give the
+// barrier phases: tile0 = K/V tiles this CTA loaded before the item, item_no
+// = prefill items before it, sph[e] = S/P phases head slot e completed.
 // ---------------------------------------------------------------------------
-__device__ void prefill_item(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem,
-                             const PrefillInfo &pf, int t, int hq, int kt0, int kt1, int part_slot,
-                             uint32_t tile0, uint32_t item_no)
+struct PrefillArgs {
+    int f, t, hq0, nh, s, ns, kt0, kt1, part_base;
+    uint32_t tile0, item_no, sph0, sph1;
+};
+
+__device__ __forceinline__ PrefillArgs prefill_args(const int4 it, const Misc *misc, uint32_t tile_cnt,
+                                                    uint32_t item_no, const uint32_t (&sph)[2])
 {
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int kvh = hq / P.n_rep;
-    // tb: token index of the chunk's row 0 in q/k/v/out/slots
-    const int cs = pf.chunk_start, p = pf.p_t, tb = pf.token_base;
+    PrefillArgs a;
+    a.f = (int)(((uint32_t)it.x >> 4) & 0xFu);
+    a.nh = (int)(((uint32_t)it.x >> 8) & 1u) + 1;
+    a.t = it.y & 0xFFFF;
+    a.hq0 = it.y >> 16;
+    a.s = it.z & 0xFFFF;
+    a.ns = it.z >> 16;
+    const int nT = (misc->pre[a.f].chunk_start + kTileN - 1) / kTileN + a.t + 1;
+    a.kt0 = (int)((long long)a.s * nT / a.ns);
+    a.kt1 = (int)((long long)(a.s + 1) * nT / a.ns);
+    a.part_base = it.w;
+    a.tile0 = tile_cnt;
+    a.item_no = item_no;
+    a.sph0 = sph[0];
+    a.sph1 = sph[1];
+    return a;
+}
+
+// Warp 0 (Q and K) or warp 2 (V): the item's tiles into a ring of `nst`
+// stages; each stage waits only on its own "empty" barrier.  Cached tiles
+// are one 2-D {64,16} box per (page, head) half from the pool map (a missing
+// page reads an out-of-range row, zero filled), the chunk's own keys one 3-D
+// box per half from the k/v map.  Page ids are read four tiles (32 pages, one
+// per lane) at a time, one batch ahead: a page-table read under load takes
+// about as long as a whole tile, so it must not sit in the issue loop.
+__device__ void prefill_load_ring(const LayerParams &P, Misc *misc, const PrefillArgs &a, bool isK,
+                                  uint32_t ring, int lane)
+{
+    const PrefillInfo &pf = misc->pre[a.f];
+    const int kvh = a.hq0 / P.n_rep;
+    const int cs = pf.chunk_start, tb = pf.token_base;
     const int nA = (cs + kTileN - 1) / kTileN;
-    const int nT = kt1 - kt0;  // key tiles of this piece: global tiles kt0 + i
-    const uint32_t sbase = smem_u32(smem);
-    const uint32_t sQ = sbase + kSmemQ, sK = sbase + kSmemK, sV = sbase + kSmemV;
-    const uint32_t bar_q = smem_u32(&misc->bar_q);
+    const int nT = a.kt1 - a.kt0;
+    const int nst = isK ? kKStages : kVStages;
+    const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
+    const void *tm_in = isK ? (const void *)&P.tm_k : (const void *)&P.tm_v;
+    uint64_t *full = isK ? misc->bar_kfull : misc->bar_vfull;
+    uint64_t *empty = isK ? misc->bar_kempty : misc->bar_vempty;
     volatile int *abort = &misc->abort;
     const uint64_t tmo = P.timeout_ns;
+    const int oob_row = P.num_pages * P.hkv * kPage;
+    const int32_t *prow = P.page_table + (size_t)pf.seq * P.max_pages;
+    auto fetch_pids = [&](int i0) {
+        const int lp = (a.kt0 + i0 + (lane >> 3)) * 8 + (lane & 7);
+        int pid = -1;
+        if (i0 + (lane >> 3) < nT && lp * kPage < cs) {
+            pid = __ldg(prow + lp);
+            if (pid < 0 || pid >= P.num_pages) {
+                if (isK)
+                    flag_error(P, ERR_PAGE);
+                pid = -1;
+            }
+        }
+        return pid;
+    };
+    int pid_cur = fetch_pids(0), pid_next = fetch_pids(4);
+    for (int i = 0; i < nT; ++i) {
+        const uint32_t c = a.tile0 + i;
+        const int st = c % nst;
+        const uint32_t ph = (c / nst) & 1;
+        const int gi = a.kt0 + i;
+        if (i > 0 && (i & 3) == 0) {
+            pid_cur = pid_next;
+            pid_next = fetch_pids(i + 4);
+        }
+        int ok = 1;
+        if (lane == 0 && !mbar_wait(smem_u32(&empty[st]), ph ^ 1, abort, tmo)) {
+            set_abort(P, misc);
+            ok = 0;
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok)
+            break;
+        const uint32_t fb = smem_u32(&full[st]);
+        const uint32_t dst = ring + st * kTileBytes;
+        if (gi < nA) {
+#pragma unroll
+            for (int pg = 0; pg < 8; ++pg) {
+                const int pid = __shfl_sync(0xffffffffu, pid_cur, (i & 3) * 8 + pg);
+                if (lane == 0) {
+                    if (pg == 0)
+                        mbar_expect_tx(fb, kTileBytes);
+                    const int y = pid >= 0 ? (pid * P.hkv + kvh) * kPage : oob_row;
+                    tma_load_2d(dst + pg * 2048, tm_pool, fb, 0, y);
+                    tma_load_2d(dst + kHalfTile + pg * 2048, tm_pool, fb, 64, y);
+                }
+            }
+        } else if (lane == 0) {
+            mbar_expect_tx(fb, kTileBytes);
+            const int z = tb + kTileN * (gi - nA);
+            tma_load_3d(dst, tm_in, fb, 0, kvh, z);
+            tma_load_3d(dst + kHalfTile, tm_in, fb, 64, kvh, z);
+        }
+    }
+}
 
-    if (warp == 0 || warp == 3) {
-        // ------------------------------------------------ TMA producers
-        // warp 0 loads Q and the K tiles, warp 3 the V tiles; each waits only
-        // on its own ring's "empty" barriers.
-        const bool isK = warp == 0;
-        if (isK && lane == 0) {
-            fence_proxy_async_smem();
-            mbar_expect_tx(bar_q, kTileBytes);
-            tma_load_3d(sQ, &P.tm_q, bar_q, 0, hq, tb + kTileM * t);
-            tma_load_3d(sQ + kHalfTile, &P.tm_q, bar_q, 64, hq, tb + kTileM * t);
-        }
-        const int nst = isK ? kKStages : kVStages;
-        const uint32_t ring = isK ? sK : sV;
-        const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
-        const void *tm_in = isK ? (const void *)&P.tm_k : (const void *)&P.tm_v;
-        uint64_t *full = isK ? misc->bar_kfull : misc->bar_pfull;
-        // V stage c % 2 is free once P_{c-2} V_{c-2} has completed: the
-        // odone barrier c & 1 (one commit fewer per tile).  V_c lands on
-        // pfull c % 3, whose phase for tile c - 3 completed before that.
-        uint64_t *empty = isK ? misc->bar_sfull : misc->bar_odone;
-        const int oob_row = P.num_pages * P.hkv * kPage;
-        // Page ids of cached tiles, four tiles (32 pages, one per lane) per
-        // load, fetched one batch ahead: a page-table read under load takes
-        // about as long as a whole tile, so it must not sit in the issue loop.
-        const int32_t *prow = P.page_table + (size_t)pf.seq * P.max_pages;
-        auto fetch_pids = [&](int i0) {
-            const int lp = (kt0 + i0 + (lane >> 3)) * 8 + (lane & 7);
-            int pid = -1;
-            if (i0 + (lane >> 3) < nT && lp * kPage < cs) {
-                pid = __ldg(prow + lp);
-                if (pid < 0 || pid >= P.num_pages) {
-                    if (isK)
-                        flag_error(P, ERR_PAGE);
-                    pid = -1;
-                }
-            }
-            return pid;
-        };
-        int pid_cur = fetch_pids(0), pid_next = fetch_pids(4);
-        for (int i = 0; i < nT; ++i) {
-            const uint32_t c = tile0 + i;
-            const int st = c % nst;
-            const uint32_t ph = (c / nst) & 1;
-            const int gi = kt0 + i;
-            const bool paged = gi < nA;
-            if (i > 0 && (i & 3) == 0) {
-                pid_cur = pid_next;
-                pid_next = fetch_pids(i + 4);
-            }
-            int pids[8];
-#pragma unroll
-            for (int pg = 0; pg < 8; ++pg)
-                pids[pg] = __shfl_sync(0xffffffffu, pid_cur, (i & 3) * 8 + pg);
-            int ok = 1;
-            if (lane == 0) {
-                if (!mbar_wait(smem_u32(&empty[st]), ph ^ 1, abort, tmo)) {
-                    set_abort(P, misc);
-                    ok = 0;
-                }
-            }
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok)
-                break;
-            if (lane == 0) {
-                const uint32_t fb = smem_u32(&full[isK ? st : (int)(c % kSBuf)]);
-                const uint32_t dst = ring + st * kTileBytes;
-                mbar_expect_tx(fb, kTileBytes);
-                if (paged) {
-#pragma unroll
-                    for (int pg = 0; pg < 8; ++pg) {
-                        const int y = pids[pg] >= 0 ? (pids[pg] * P.hkv + kvh) * kPage : oob_row;
-#pragma unroll
-                        for (int hf = 0; hf < 2; ++hf)
-                            tma_load_2d(dst + hf * kHalfTile + pg * 2048, tm_pool, fb, hf * 64, y);
-                    }
-                } else {
-                    const int z = tb + kTileN * (gi - nA);
-#pragma unroll
-                    for (int hf = 0; hf < 2; ++hf)
-                        tma_load_3d(dst + hf * kHalfTile, tm_in, fb, hf * 64, kvh, z);
-                }
-            }
-        }
-    } else if (warp == 1) {
-        // ------------------------------------------------ MMA issuer
-        // One straight loop: S_i = Q K_i^T is issued before P_{i-2} V_{i-2}
-        // (three S buffers), so the softmax of tile i - 1 and i runs while
-        // the tensor pipe works on P.V of i - 2 and S of i.  The descriptors
-        // are formed once per tile and advanced by constants.  A wait issued
-        // behind queued MMAs returns only once they have been accepted (the
-        // tensor pipe drains and refills), so each MMA group costs one such
-        // boundary and the commits are kept to a minimum.
-        if (lane == 0) {
-            bool ok = mbar_wait(bar_q, item_no & 1, abort, tmo);
-            tc_fence_after();
-            const uint64_t qdesc = smem_desc(sQ, 16, 1024, kSwz128);
-            for (int i = 0; ok && i < nT + 2; ++i) {
-                if (i < nT) {
-                    const uint32_t c = tile0 + i;
-                    const int st = c % kKStages;
-                    if (!mbar_wait(smem_u32(&misc->bar_kfull[st]), (c / kKStages) & 1, abort, tmo)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint64_t kdesc = smem_desc(sK + st * kTileBytes, 16, 1024, kSwz128);
-                    const uint32_t d = tmem + (c % kSBuf) * 128;
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        // 16 dims of K-major SW128: +32 B inside a 64-column half
-                        const uint64_t off = (uint64_t)(((kk >> 2) * kHalfTile + (kk & 3) * 32) >> 4);
-                        tc_mma_ss(d, qdesc + off, kdesc + off, kIdescS, kk > 0 ? 1u : 0u);
-                    }
-                    tc_commit(smem_u32(&misc->bar_sfull[c % kSBuf]));  // also frees K stage st
-                }
-                if (i >= 2) {
-                    const int j = i - 2;
-                    const uint32_t c = tile0 + j;
-                    const int st = c % kVStages;
-                    if (!mbar_wait(smem_u32(&misc->bar_pfull[c % kSBuf]), (c / kSBuf) & 1, abort, tmo)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t dv = sV + st * kTileBytes;
-                    if (kt0 + j == nA - 1 && (cs % kTileN) != 0)
-                        clear_uncached_rows(dv, cs - (kt0 + j) * kTileN);
-                    tc_fence_after();
-                    const uint64_t vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
-                    const uint32_t pa = tmem + (c % kSBuf) * 128;  // P_c over S_c: 8 columns per 16 keys
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk)  // 16 keys of MN-major V: +2 KiB
-                        tc_mma_ts(tmem + kTmemO, pa + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4), kIdescO,
-                                  (j > 0 || kk > 0) ? 1u : 0u);
-                    if (false) {  // the low-order part of P
-#pragma unroll
-                        for (int kk = 0; kk < 8; ++kk)
-                            tc_mma_ts(tmem + kTmemO, pa + 64 + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4),
-                                      kIdescO, 1u);
-                    }
-                    tc_commit(smem_u32(&misc->bar_odone[c & 1]));  // also frees V stage st
-                }
-            }
-            if (!ok)
-                set_abort(P, misc);
-        }
-        __syncwarp();
-    } else if (warp >= 4) {
-        // ------------------------------------------------ softmax / epilogue
-        const int q4 = warp - 4;
-        const int r = q4 * 32 + lane;          // tile row = TMEM lane
-        const int j = kTileM * t + r;          // chunk row offset
-        const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
-        const float sl = P.scale_log2;
-        {
-            // Piece 0 appends this head's share of the tile's K/V: the n_rep
-            // query heads of a KV head split its 128 tokens (head r of the
-            // group takes tokens [r*128/n_rep, (r+1)*128/n_rep)), and the 32
-            // 16-byte pieces of a token's K and V rows are split between
-            // n_rep threads; all loads are in flight at once (two rounds for
-            // n_rep = 1), while Q and the first K tile land.
-            const int per = kTileM / P.n_rep, npc = 32 / P.n_rep;
-            const int u = r / P.n_rep, sub = r % P.n_rep;
-            const int ja = kTileM * t + (hq % P.n_rep) * per + u;   // chunk row of this thread's token
-            const bool app = kt0 == 0 && ja < p;
-            const size_t arow = ((size_t)(tb + ja) * P.hkv + kvh) * kHeadDim;
-            int slot = -1;
-            if (app)
-                slot = __ldg(P.slots + tb + ja);
-            for (int b = 0; app && b < npc; b += 16) {
-                uint4 av[16];
-#pragma unroll
-                for (int x = 0; x < 16; ++x) {
-                    const int pc = sub * npc + b + x;   // piece: K row 0..15, V row 16..31
-                    if (x < npc - b)
-                        av[x] = __ldg(reinterpret_cast<const uint4 *>((pc < 16 ? P.k : P.v) + arow) + (pc & 15));
-                }
-                if (slot >= P.num_pages * kPage) {
-                    if (sub == 0 && b == 0)
-                        flag_error(P, ERR_SLOT);
-                } else if (slot >= 0) {
-                    const size_t dst = (((size_t)(slot / kPage) * P.hkv + kvh) * kPage + slot % kPage) * kHeadDim;
-#pragma unroll
-                    for (int x = 0; x < 16; ++x) {
-                        const int pc = sub * npc + b + x;
-                        if (x < npc - b)
-                            reinterpret_cast<uint4 *>((pc < 16 ? P.k_pool : P.v_pool) + dst)[pc & 15] = av[x];
-                    }
-                }
-            }
-        }
-        float m_run = neg_inf(), l_run = 0.f;
-        bool ok = true;
-        for (int i = 0; i < nT; ++i) {
-            const uint32_t c = tile0 + i;
-            const int sb = c % kSBuf;
-            if (!mbar_wait(smem_u32(&misc->bar_sfull[sb]), (c / kSBuf) & 1, abort, tmo)) {
+// Warp 1, one thread: every MMA of the item.  Per key tile j (the loop runs
+// one step past the last tile for the final P.V):
+//   [P_0(j-1) written]  O_0 += P_0 V_{j-1}   [K_j landed]  S_0 = Q_0 K_j -> sfull[0]
+//   [P_1(j-1) written]  O_1 += P_1 V_{j-1}                 S_1 = Q_1 K_j -> sfull[1]
+//   -> kempty (K_j free), vempty (V_{j-1} free)
+// so the softmax of head 0 for tile j runs while the tensor pipe works on
+// head 1's P.V and S, and the other way round.  S_h = Q_h K_j overwrites the
+// TMEM columns that P_h(j-1) occupied; it is issued after P_h(j-1) V_{j-1},
+// and the pipe executes in order.  A commit covers every earlier MMA of the
+// thread, so sfull[h] of tile j also says that O_h += P_h V_{j-1} is done.
+__device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs &a, uint32_t tmem,
+                            uint32_t sbase)
+{
+    const PrefillInfo &pf = misc->pre[a.f];
+    const int cs = pf.chunk_start;
+    const int nA = (cs + kTileN - 1) / kTileN;
+    const int nT = a.kt1 - a.kt0;
+    volatile int *abort = &misc->abort;
+    const uint64_t tmo = P.timeout_ns;
+    const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;
+    bool ok = mbar_wait(smem_u32(&misc->bar_q), a.item_no & 1, abort, tmo);
+    tc_fence_after();
+    const uint64_t qd0 = smem_desc(sbase + kSmemQ, 16, 1024, kSwz128);
+    const uint64_t qd1 = smem_desc(sbase + kSmemQ + kTileBytes, 16, 1024, kSwz128);
+    for (int j = 0; ok && j <= nT; ++j) {
+        const uint32_t c = a.tile0 + j;
+        uint64_t vdesc = 0;
+        if (j > 0) {
+            const uint32_t cp = c - 1;
+            if (!mbar_wait(smem_u32(&misc->bar_vfull[cp % kVStages]), (cp / kVStages) & 1, abort, tmo)) {
                 ok = false;
                 break;
             }
-            tc_fence_after();
-            const int gi = kt0 + i;
-            const int nvalid = gi < nA ? min(kTileN, cs - gi * kTileN)
-                                       : min(kTileN, j - kTileN * (gi - nA) + 1);
-            // Row r of S_c: all 128 raw scores read from TMEM once (a second
-            // read would compete with the tensor core's own TMEM traffic).
-            uint32_t sv[128];
+            const uint32_t dv = sV + (cp % kVStages) * kTileBytes;
+            if (a.kt0 + j - 1 == nA - 1 && (cs % kTileN) != 0)
+                clear_uncached_rows(dv, cs - (a.kt0 + j - 1) * kTileN);
+            vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
+            asm volatile("" : "+l"(vdesc));
+        }
+        uint64_t kdesc = 0;
+        bool kready = false;
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-                tmem_ld32(tl + sb * 128 + 32 * q, *reinterpret_cast<uint32_t(*)[32]>(&sv[32 * q]));
-            tmem_wait_ld();
-            if (nvalid < kTileN) {  // boundary tiles only: masked keys -> -inf
-#pragma unroll
-                for (int cc = 0; cc < 128; ++cc)
-                    if (cc >= nvalid)
-                        sv[cc] = 0xFF800000u;
-            }
-            const float mx = row_max(sv);
-            const float m_new = fmaxf(m_run, mx * sl);   // log2 domain
-            const bool rescale = m_new > m_run + 8.0f;
-            const float m_use = rescale ? m_new : m_run;
-            const float nm = -m_use;
-            // P_c (the A operand of P.V) goes over the first 64 columns of
-            // S_c, whose buffer P_{c-3} held: S_c was issued after
-            // P_{c-3} V_{c-3}, so its completion covers that read too.
-            // rows with fewer than 17 keys (the first rows of a prompt) take P as hi + lo
-            const float rs = row_exp_store(sv, sl, nm, tl + sb * 128, false);
-            // The O correction comes after P, when the scores are no longer
-            // live, and before P_c is released to the MMA issuer.
-            if (rescale && i > 0) {
-                // O must be stable: tile c - 1's PV has completed.
-                if (!mbar_wait(smem_u32(&misc->bar_odone[(c - 1) & 1]), ((c - 1) >> 1) & 1, abort, tmo)) {
+        for (int e = 0; e < 2; ++e) {
+            if (e >= a.nh)
+                break;
+            if (j > 0) {
+                // O_e += P_e(j-1) V_{j-1}, as soon as head e's softmax wrote P
+                if (!mbar_wait(smem_u32(&misc->bar_pfull[e]), ((e == 0 ? a.sph0 : a.sph1) + j - 1) & 1, abort,
+                               tmo)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const float alpha = ex2(m_run - m_use);
+                const uint32_t pa = tmem + kTmemS + e * 128;   // P_e: 8 columns per 16 keys
 #pragma unroll
-                for (int gq = 0; gq < 4; ++gq) {
-                    uint32_t o[32];
-                    tmem_ld32(tl + kTmemO + 32 * gq, o);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int x = 0; x < 32; ++x)
-                        o[x] = __float_as_uint(__uint_as_float(o[x]) * alpha);
-                    tmem_st32(tl + kTmemO + 32 * gq, o);
-                }
-                tmem_wait_st();
-                l_run *= alpha;
+                for (int kk = 0; kk < 8; ++kk)   // 16 keys of MN-major V: +2 KiB
+                    tc_mma_ts(tmem + kTmemO + e * 128, pa + kk * 8, vdesc + (uint64_t)((kk * 2048) >> 4),
+                              kIdescO, (j > 1 || kk > 0) ? 1u : 0u);
             }
-            l_run += rs;
-            m_run = m_use;
-            tmem_wait_st();
-            tc_fence_before();
-            mbar_arrive(smem_u32(&misc->bar_pfull[sb]));
-        }
-        if (ok) {
-            // O is complete after the last P.V.  Its odone barrier may still
-            // be one phase behind (P_{cl-2} V_{cl-2} in flight: S_cl only
-            // covers P_{cl-3} V_{cl-3}), so P_{cl-1} V_{cl-1} is awaited
-            // first; a parity wait is unambiguous only one phase ahead.
-            const uint32_t cl = tile0 + nT - 1;
-            if (!mbar_wait(smem_u32(&misc->bar_odone[(cl - 1) & 1]), ((cl - 1) >> 1) & 1, abort, tmo) ||
-                !mbar_wait(smem_u32(&misc->bar_odone[cl & 1]), (cl >> 1) & 1, abort, tmo))
-                ok = false;
-        }
-        if (!ok) {
-            set_abort(P, misc);
-        } else if (part_slot >= 0) {
-            // one piece of a split tile: normalised partial O and its lse
-            tc_fence_after();
-            const float inv = 1.0f / l_run;
-            float *prow = P.pre_o + ((size_t)part_slot * kTileM + r) * kHeadDim;
-#pragma unroll
-            for (int gq = 0; gq < 4; ++gq) {
-                uint32_t o[32];
-                tmem_ld32(tl + kTmemO + 32 * gq, o);
-                tmem_wait_ld();
-#pragma unroll
-                for (int x = 0; x < 8; ++x)
-                    reinterpret_cast<float4 *>(prow + 32 * gq)[x] =
-                        make_float4(__uint_as_float(o[4 * x]) * inv, __uint_as_float(o[4 * x + 1]) * inv,
-                                    __uint_as_float(o[4 * x + 2]) * inv, __uint_as_float(o[4 * x + 3]) * inv);
-            }
-            float lg;
-            asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(lg) : "f"(l_run));
-            P.pre_lse[(size_t)part_slot * kTileM + r] = m_run + lg;
-            __threadfence();
-        } else {
-            tc_fence_after();
-            const float inv = 1.0f / l_run;
-            uint16_t *orow = P.out + ((size_t)(tb + j) * P.hq + hq) * kHeadDim;
-#pragma unroll
-            for (int gq = 0; gq < 4; ++gq) {
-                uint32_t o[32];
-                tmem_ld32(tl + kTmemO + 32 * gq, o);
-                tmem_wait_ld();
-                if (j < p) {
-#pragma unroll
-                    for (int x = 0; x < 4; ++x) {
-                        uint4 v4;
-                        v4.x = pack_bf16(__uint_as_float(o[8 * x + 0]) * inv, __uint_as_float(o[8 * x + 1]) * inv);
-                        v4.y = pack_bf16(__uint_as_float(o[8 * x + 2]) * inv, __uint_as_float(o[8 * x + 3]) * inv);
-                        v4.z = pack_bf16(__uint_as_float(o[8 * x + 4]) * inv, __uint_as_float(o[8 * x + 5]) * inv);
-                        v4.w = pack_bf16(__uint_as_float(o[8 * x + 6]) * inv, __uint_as_float(o[8 * x + 7]) * inv);
-                        reinterpret_cast<uint4 *>(orow + 32 * gq)[x] = v4;
+            if (j < nT) {
+                if (!kready) {
+                    if (!mbar_wait(smem_u32(&misc->bar_kfull[c % kKStages]), (c / kKStages) & 1, abort, tmo)) {
+                        ok = false;
+                        break;
                     }
+                    tc_fence_after();
+                    kdesc = smem_desc(sK + (c % kKStages) * kTileBytes, 16, 1024, kSwz128);
+                    asm volatile("" : "+l"(kdesc));
+                    kready = true;
                 }
+                // S_e(j) = Q_e K_j^T.  Opaque per tile, so that the compiler
+                // does not keep the 8 offset descriptors of both heads live
+                // across the loop.
+                uint64_t qd = e == 0 ? qd0 : qd1;
+                asm volatile("" : "+l"(qd));
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    // 16 dims of K-major SW128: +32 B inside a 64-column half
+                    const uint64_t off = (uint64_t)(((kk >> 2) * kHalfTile + (kk & 3) * 32) >> 4);
+                    tc_mma_ss(tmem + kTmemS + e * 128, qd + off, kdesc + off, kIdescS, kk > 0 ? 1u : 0u);
+                }
+                tc_commit(smem_u32(&misc->bar_sfull[e]));
             }
-            // the first 16 rows of a prompt: exact fp32 recomputation (the
-            // item has one key tile, tile0's K and V stages hold it)
-            if (cs == 0 && t == 0 && r < kPage && j < p) {
-                // the tiles' TMA writes, observed on their own (completed) barriers
-                if (mbar_wait(bar_q, item_no & 1, abort, tmo) &&
-                    mbar_wait(smem_u32(&misc->bar_kfull[tile0 % kKStages]), (tile0 / kKStages) & 1, abort, tmo) &&
-                    mbar_wait(smem_u32(&misc->bar_pfull[tile0 % kSBuf]), (tile0 / kSBuf) & 1, abort, tmo))
-                    short_row_exact(sQ, sK + (tile0 % kKStages) * kTileBytes, sV + (tile0 % kVStages) * kTileBytes,
-                                    r, sl, orow);
+        }
+        if (!ok)
+            break;
+        if (j < nT)
+            tc_commit(smem_u32(&misc->bar_kempty[c % kKStages]));
+        if (j > 0)
+            tc_commit(smem_u32(&misc->bar_vempty[(c - 1) % kVStages]));
+    }
+    if (ok)
+        tc_commit(smem_u32(&misc->bar_odone));
+    else
+        set_abort(P, misc);
+}
+
+// Piece 0 of each of the n_rep / nh items of a KV head appends its share of
+// the tile's tokens (item r of the group takes tokens [r*128/(n_rep/nh),
+// (r+1)*128/(n_rep/nh))); the 32 16-byte pieces of a token's K and V rows are
+// spread over the 256 consumer threads, all loads in flight at once, while Q
+// and the first K tile land.
+__device__ __forceinline__ void prefill_append(const LayerParams &P, const PrefillInfo &pf, const PrefillArgs &a,
+                                               int tid)
+{
+    const int groups = P.n_rep / a.nh;              // items per KV head and tile
+    const int per = kTileM / groups;                // tokens of this item
+    const int kvh = a.hq0 / P.n_rep;
+    const int r0 = kTileM * a.t + ((a.hq0 % P.n_rep) / a.nh) * per;   // first chunk row
+    const int n_pc = per * 32;                      // 16-byte pieces
+    constexpr int kRound = 8;                       // loads in flight per thread
+#pragma unroll 1
+    for (int b = 0; b < n_pc; b += kRound * kConsThreads) {
+        uint4 av[kRound];
+        int slot[kRound];
+#pragma unroll
+        for (int x = 0; x < kRound; ++x) {
+            const int pc = b + tid + kConsThreads * x;
+            const int u = pc >> 5, w = pc & 31;
+            slot[x] = -1;
+            if (pc < n_pc && r0 + u < pf.p_t) {
+                const size_t src = ((size_t)(pf.token_base + r0 + u) * P.hkv + kvh) * kHeadDim;
+                slot[x] = __ldg(P.slots + pf.token_base + r0 + u);
+                av[x] = __ldg(reinterpret_cast<const uint4 *>((w < 16 ? P.k : P.v) + src) + (w & 15));
+            }
+        }
+#pragma unroll
+        for (int x = 0; x < kRound; ++x) {
+            const int w = (b + tid + kConsThreads * x) & 31;
+            const int sl = slot[x];
+            if (sl >= P.num_pages * kPage) {
+                if (w == 0)
+                    flag_error(P, ERR_SLOT);
+            } else if (sl >= 0) {
+                const size_t dst = (((size_t)(sl / kPage) * P.hkv + kvh) * kPage + sl % kPage) * kHeadDim;
+                reinterpret_cast<uint4 *>((w < 16 ? P.k_pool : P.v_pool) + dst)[w & 15] = av[x];
             }
         }
     }
 }
 
-// Merge the n_s pieces of prefill tile (t, hq) if this CTA's piece arrived
-// last (no waiting): out = sum_s w_s O_s / sum_s w_s, w_s = 2^(lse_s - max).
-__device__ void prefill_merge(const LayerParams &P, Misc *misc, const PrefillInfo &pf, int t, int hq,
-                              int n_s, int part_base)
+// Consumer warpgroup e (its 128 threads, TMEM lane = row): the softmax of
+// query head hq0 + e over the item's key tiles, then its epilogue.
+__device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc, const PrefillArgs &a,
+                                uint32_t tmem, int e, int r)
 {
-    const int tid = threadIdx.x;
-    if (tid == 0) {
-        const uint32_t prev = atomicAdd(P.pre_cnt + (pf.tile_base + t) * P.hq + hq, 1u);
-        misc->last = (prev == (uint32_t)(n_s - 1)) ? 1 : 0;
-    }
-    __syncthreads();
-    if (misc->last) {
-        __threadfence();
-        const int r = tid >> 1, half = tid & 1;
-        const int j = kTileM * t + r;
-        if (j < pf.p_t) {
-            float M = neg_inf();
-            for (int s = 0; s < n_s; ++s)
-                M = fmaxf(M, __ldcg(P.pre_lse + (size_t)(part_base + s) * kTileM + r));
-            float W = 0.f;
-            for (int s = 0; s < n_s; ++s)
-                W += ex2(__ldcg(P.pre_lse + (size_t)(part_base + s) * kTileM + r) - M);
-            const float inv = 1.0f / W;
-            for (int sub = 0; sub < 2; ++sub) {
-                const int d0 = half * 64 + sub * 32;
-                float acc[32];
+    const PrefillInfo &pf = misc->pre[a.f];
+    const int cs = pf.chunk_start, p = pf.p_t, tb = pf.token_base;
+    const int nA = (cs + kTileN - 1) / kTileN;
+    const int nT = a.kt1 - a.kt0;
+    const int hq = a.hq0 + e;
+    const int j = kTileM * a.t + r;          // chunk row offset
+    const int q4 = r >> 5;
+    const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
+    const uint32_t tS = tl + kTmemS + e * 128, tO = tl + kTmemO + e * 128;
+    const uint32_t sbase = smem_u32(smem);
+    const float sl = P.scale_log2;
+    const uint32_t ph0 = e == 0 ? a.sph0 : a.sph1;
+    volatile int *abort = &misc->abort;
+    const uint64_t tmo = P.timeout_ns;
+
+    float m_run = neg_inf(), l_run = 0.f;
+    bool ok = true;
+    for (int i = 0; i < nT; ++i) {
+        if (!mbar_wait(smem_u32(&misc->bar_sfull[e]), (ph0 + i) & 1, abort, tmo)) {
+            ok = false;
+            break;
+        }
+        tc_fence_after();
+        const int gi = a.kt0 + i;
+        const int nvalid = gi < nA ? min(kTileN, cs - gi * kTileN) : min(kTileN, j - kTileN * (gi - nA) + 1);
+        // Row r of S: all 128 raw scores read from TMEM once (a second read
+        // would compete with the tensor core's own TMEM traffic).
+        uint32_t sv[128];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            tmem_ld32(tS + 32 * q, *reinterpret_cast<uint32_t(*)[32]>(&sv[32 * q]));
+        tmem_wait_ld();
+        if (nvalid < kTileN) {  // boundary tiles only: masked keys -> -inf
+#pragma unroll
+            for (int cc = 0; cc < 128; ++cc)
+                if (cc >= nvalid)
+                    sv[cc] = 0xFF800000u;
+        }
+        const float mx = row_max(sv);
+        const float m_new = fmaxf(m_run, mx * sl);   // log2 domain
+        const bool rescale = m_new > m_run + 8.0f;
+        const float m_use = rescale ? m_new : m_run;
+        // P over the first 64 columns of S (the A operand of P.V)
+        const float rs = row_exp_store(sv, sl, -m_use, tS);
+        // FA4-style lazy rescale: O moves only when the row max grows by more
+        // than 8 in log2 units.  O_e is stable here: sfull of this tile was
+        // committed after O_e += P_e V of the previous tile, and the next P.V
+        // waits for this tile's P.
+        if (rescale && i > 0) {
+            const float alpha = ex2(m_run - m_use);
+#pragma unroll
+            for (int gq = 0; gq < 4; ++gq) {
+                uint32_t o[32];
+                tmem_ld32(tO + 32 * gq, o);
+                tmem_wait_ld();
 #pragma unroll
                 for (int x = 0; x < 32; ++x)
-                    acc[x] = 0.f;
-                for (int s = 0; s < n_s; ++s) {
-                    const float w = ex2(__ldcg(P.pre_lse + (size_t)(part_base + s) * kTileM + r) - M);
-                    const float4 *src = reinterpret_cast<const float4 *>(
-                        P.pre_o + ((size_t)(part_base + s) * kTileM + r) * kHeadDim + d0);
+                    o[x] = __float_as_uint(__uint_as_float(o[x]) * alpha);
+                tmem_st32(tO + 32 * gq, o);
+            }
+            l_run *= alpha;
+        }
+        l_run += rs;
+        m_run = m_use;
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(smem_u32(&misc->bar_pfull[e]));
+    }
+    if (ok && !mbar_wait(smem_u32(&misc->bar_odone), a.item_no & 1, abort, tmo))
+        ok = false;
+    if (!ok) {
+        set_abort(P, misc);
+        return;
+    }
+    tc_fence_after();
+    const float inv = 1.0f / l_run;
+    if (a.ns > 1) {
+        // one piece of a split tile: normalised partial O and its lse
+        const int part_slot = a.part_base + e * a.ns + a.s;
+        float *prow = P.pre_o + ((size_t)part_slot * kTileM + r) * kHeadDim;
 #pragma unroll
-                    for (int x = 0; x < 8; ++x) {
-                        const float4 v = __ldcg(src + x);
-                        acc[4 * x] += w * v.x;
-                        acc[4 * x + 1] += w * v.y;
-                        acc[4 * x + 2] += w * v.z;
-                        acc[4 * x + 3] += w * v.w;
-                    }
-                }
-                uint4 *dst = reinterpret_cast<uint4 *>(
-                    P.out + ((size_t)(pf.token_base + j) * P.hq + hq) * kHeadDim + d0);
+        for (int gq = 0; gq < 4; ++gq) {
+            uint32_t o[32];
+            tmem_ld32(tO + 32 * gq, o);
+            tmem_wait_ld();
 #pragma unroll
-                for (int x = 0; x < 4; ++x)
-                    dst[x] = make_uint4(pack_bf16(acc[8 * x] * inv, acc[8 * x + 1] * inv),
-                                        pack_bf16(acc[8 * x + 2] * inv, acc[8 * x + 3] * inv),
-                                        pack_bf16(acc[8 * x + 4] * inv, acc[8 * x + 5] * inv),
-                                        pack_bf16(acc[8 * x + 6] * inv, acc[8 * x + 7] * inv));
+            for (int x = 0; x < 8; ++x)
+                reinterpret_cast<float4 *>(prow + 32 * gq)[x] =
+                    make_float4(__uint_as_float(o[4 * x]) * inv, __uint_as_float(o[4 * x + 1]) * inv,
+                                __uint_as_float(o[4 * x + 2]) * inv, __uint_as_float(o[4 * x + 3]) * inv);
+        }
+        float lg;
+        asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(lg) : "f"(l_run));
+        P.pre_lse[(size_t)part_slot * kTileM + r] = m_run + lg;
+        __threadfence();
+        return;
+    }
+    uint16_t *orow = P.out + ((size_t)(tb + j) * P.hq + hq) * kHeadDim;
+#pragma unroll
+    for (int gq = 0; gq < 4; ++gq) {
+        uint32_t o[32];
+        tmem_ld32(tO + 32 * gq, o);
+        tmem_wait_ld();
+        if (j < p) {
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                uint4 v4;
+                v4.x = pack_bf16(__uint_as_float(o[8 * x + 0]) * inv, __uint_as_float(o[8 * x + 1]) * inv);
+                v4.y = pack_bf16(__uint_as_float(o[8 * x + 2]) * inv, __uint_as_float(o[8 * x + 3]) * inv);
+                v4.z = pack_bf16(__uint_as_float(o[8 * x + 4]) * inv, __uint_as_float(o[8 * x + 5]) * inv);
+                v4.w = pack_bf16(__uint_as_float(o[8 * x + 6]) * inv, __uint_as_float(o[8 * x + 7]) * inv);
+                reinterpret_cast<uint4 *>(orow + 32 * gq)[x] = v4;
             }
         }
-        if (tid == 0)
-            P.pre_cnt[t * P.hq + hq] = 0u;
     }
-    __syncthreads();
+    // rows with at most 16 keys (positions 0..15 of a prompt): exact fp32
+    // recomputation.  The item (t = 0, never split) has one key tile (cs = 0)
+    // or two (0 < cs < 16: the cached tile, then the chunk's own), all still
+    // in their K and V stages (at least two of each).
+    if (a.t == 0 && cs < kPage && cs + r < kPage && j < p) {
+        const uint32_t ca = a.tile0, cb = a.tile0 + (cs > 0 ? 1u : 0u);
+        static_assert(kKStages >= 2 && kVStages >= 2, "the short rows need two tiles in the rings");
+        const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;
+        // the tiles' TMA writes, observed on their own (completed) barriers
+        if (mbar_wait(smem_u32(&misc->bar_q), a.item_no & 1, abort, tmo) &&
+            mbar_wait(smem_u32(&misc->bar_kfull[ca % kKStages]), (ca / kKStages) & 1, abort, tmo) &&
+            mbar_wait(smem_u32(&misc->bar_vfull[ca % kVStages]), (ca / kVStages) & 1, abort, tmo) &&
+            mbar_wait(smem_u32(&misc->bar_kfull[cb % kKStages]), (cb / kKStages) & 1, abort, tmo) &&
+            mbar_wait(smem_u32(&misc->bar_vfull[cb % kVStages]), (cb / kVStages) & 1, abort, tmo))
+            short_row_exact(sbase + kSmemQ + e * kTileBytes, sK + (ca % kKStages) * kTileBytes,
+                            sV + (ca % kVStages) * kTileBytes, sK + (cb % kKStages) * kTileBytes,
+                            sV + (cb % kVStages) * kTileBytes, cs, r, sl, orow);
+    }
+}
+
+// Merge the n_s pieces of prefill tile (t, hq0 .. hq0 + nh - 1) if this CTA's
+// piece arrived last (no waiting): out = sum_s w_s O_s / sum_s w_s,
+// w_s = 2^(lse_s - max).  Run by the 256 consumer threads.
+__device__ void prefill_merge(const LayerParams &P, Misc *misc, const PrefillInfo &pf, const PrefillArgs &a,
+                              int tid)
+{
+    // the tile's arrival counter, indexed over the query tiles of all chunks
+    uint32_t *cnt = P.pre_cnt + (size_t)(pf.tile_base + a.t) * P.hq + a.hq0;
+    cons_sync();   // every consumer thread's partial is written (and fenced)
+    if (tid == 0) {
+        const uint32_t prev = atomicAdd(cnt, 1u);
+        misc->last = (prev == (uint32_t)(a.ns - 1)) ? 1 : 0;
+    }
+    cons_sync();
+    if (!misc->last)
+        return;
+    __threadfence();
+    const int r = tid >> 1, half = tid & 1;
+    const int j = kTileM * a.t + r;
+    for (int e = 0; e < a.nh && j < pf.p_t; ++e) {
+        const int base = a.part_base + e * a.ns;
+        float M = neg_inf();
+        for (int s = 0; s < a.ns; ++s)
+            M = fmaxf(M, __ldcg(P.pre_lse + (size_t)(base + s) * kTileM + r));
+        float W = 0.f;
+        for (int s = 0; s < a.ns; ++s)
+            W += ex2(__ldcg(P.pre_lse + (size_t)(base + s) * kTileM + r) - M);
+        const float inv = 1.0f / W;
+        for (int sub = 0; sub < 2; ++sub) {
+            const int d0 = half * 64 + sub * 32;
+            float acc[32];
+#pragma unroll
+            for (int x = 0; x < 32; ++x)
+                acc[x] = 0.f;
+            for (int s = 0; s < a.ns; ++s) {
+                const float w = ex2(__ldcg(P.pre_lse + (size_t)(base + s) * kTileM + r) - M);
+                const float4 *src =
+                    reinterpret_cast<const float4 *>(P.pre_o + ((size_t)(base + s) * kTileM + r) * kHeadDim + d0);
+#pragma unroll
+                for (int x = 0; x < 8; ++x) {
+                    const float4 v = __ldcg(src + x);
+                    acc[4 * x] += w * v.x;
+                    acc[4 * x + 1] += w * v.y;
+                    acc[4 * x + 2] += w * v.z;
+                    acc[4 * x + 3] += w * v.w;
+                }
+            }
+            uint4 *dst = reinterpret_cast<uint4 *>(P.out + ((size_t)(pf.token_base + j) * P.hq + a.hq0 + e) *
+                                                              kHeadDim + d0);
+#pragma unroll
+            for (int x = 0; x < 4; ++x)
+                dst[x] = make_uint4(pack_bf16(acc[8 * x] * inv, acc[8 * x + 1] * inv),
+                                    pack_bf16(acc[8 * x + 2] * inv, acc[8 * x + 3] * inv),
+                                    pack_bf16(acc[8 * x + 4] * inv, acc[8 * x + 5] * inv),
+                                    pack_bf16(acc[8 * x + 6] * inv, acc[8 * x + 7] * inv));
+        }
+    }
+    if (tid == 0)
+        *cnt = 0u;
+}
+
+// Between items: every thread of the CTA has finished the previous item.
+__device__ __forceinline__ void item_boundary()
+{
+    tc_fence_before();
+    named_sync(kBarItem, kThreads);
+    tc_fence_after();
+}
+
+// Warpgroup 0's item loop: claims the next item, loads tiles, issues MMAs.
+__device__ void producer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t sbase = smem_u32(smem);
+    uint32_t tile_cnt = 0, item_no = 0, sph[2] = {0u, 0u};
+    int buf = 0;
+    for (;;) {
+        item_boundary();
+        const int idx = misc->item_idx[buf];
+        if (idx >= P.n_items || misc->abort)
+            break;
+        if (tid == 0)
+            misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
+        const int4 it = P.items[idx];
+        if ((it.x & 0xF) == ITEM_PREFILL) {
+            const PrefillArgs a = prefill_args(it, misc, tile_cnt, item_no, sph);
+            if (warp == 0) {
+                if (lane == 0) {
+                    // Q of the item's heads (the previous item's MMAs and
+                    // short rows are done: every thread passed the boundary)
+                    fence_proxy_async_smem();
+                    const uint32_t bq = smem_u32(&misc->bar_q);
+                    const PrefillInfo &pf = misc->pre[a.f];
+                    mbar_expect_tx(bq, a.nh * kTileBytes);
+                    for (int e = 0; e < a.nh; ++e) {
+                        const uint32_t dq = sbase + kSmemQ + e * kTileBytes;
+                        tma_load_3d(dq, &P.tm_q, bq, 0, a.hq0 + e, pf.token_base + kTileM * a.t);
+                        tma_load_3d(dq + kHalfTile, &P.tm_q, bq, 64, a.hq0 + e, pf.token_base + kTileM * a.t);
+                    }
+                }
+                prefill_load_ring(P, misc, a, true, sbase + kSmemK, lane);
+            } else if (warp == 2) {
+                prefill_load_ring(P, misc, a, false, sbase + kSmemV, lane);
+            } else if (warp == 1 && lane == 0) {
+                prefill_mma(P, misc, a, tmem, sbase);
+            }
+            const uint32_t nT = (uint32_t)(a.kt1 - a.kt0);
+            tile_cnt += nT;
+            item_no += 1;
+            sph[0] += nT;
+            if (a.nh == 2)
+                sph[1] += nT;
+        }
+        __syncwarp();
+        buf ^= 1;
+    }
+}
+
+// The consumer warpgroups' item loop: softmax and epilogue of prefill items,
+// all of a decode item.
+__device__ void consumer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem)
+{
+    const int tid = threadIdx.x - kProdThreads;     // 0..255
+    uint32_t tile_cnt = 0, item_no = 0, sph[2] = {0u, 0u};
+    int buf = 0;
+    for (;;) {
+        item_boundary();
+        const int idx = misc->item_idx[buf];
+        if (idx >= P.n_items || misc->abort)
+            break;
+        const int4 it = P.items[idx];
+        if ((it.x & 0xF) == ITEM_PREFILL) {
+            const PrefillArgs a = prefill_args(it, misc, tile_cnt, item_no, sph);
+            const PrefillInfo &pf = misc->pre[a.f];
+            if (a.kt0 == 0)
+                prefill_append(P, pf, a, tid);
+            const int e = tid >> 7;
+            if (e < a.nh)
+                prefill_softmax(P, smem, misc, a, tmem, e, tid & 127);
+            // every consumer thread takes part in the merge's barriers, also
+            // after an abort (the merge then writes what it finds; the call
+            // reports the error and the host clears the counters)
+            if (a.ns > 1)
+                prefill_merge(P, misc, pf, a, tid);
+            const uint32_t nT = (uint32_t)(a.kt1 - a.kt0);
+            tile_cnt += nT;
+            item_no += 1;
+            sph[0] += nT;
+            if (a.nh == 2)
+                sph[1] += nT;
+        } else if ((it.x & 0xF) == ITEM_DECODE_SHORT) {
+            decode_short_item(P, smem, it.y, (int)(((uint32_t)it.x >> 4) & 0x7Fu), it.z, it.w, tid);
+        } else {
+            const uint32_t dx = (uint32_t)it.x;
+            decode_item(P, smem, misc, it.y, (int)((dx >> 4) & 0x7Fu), (int)((dx >> 11) & 0xFFFu), it.z, it.w,
+                        (int)(dx >> 23) * 16, tid);
+        }
+        fence_proxy_async_smem();  // generic smem accesses before later TMA writes
+        buf ^= 1;
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -1030,13 +1178,17 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         mbar_init(smem_u32(&misc->bar_q), 1);
         for (int b = 0; b < kKStages; ++b) {
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
+            mbar_init(smem_u32(&misc->bar_kempty[b]), 1);
         }
-        for (int b = 0; b < kSBuf; ++b) {
+        for (int b = 0; b < kVStages; ++b) {
+            mbar_init(smem_u32(&misc->bar_vfull[b]), 1);
+            mbar_init(smem_u32(&misc->bar_vempty[b]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&misc->bar_sfull[b]), 1);
-            mbar_init(smem_u32(&misc->bar_pfull[b]), 128 + 1);
+            mbar_init(smem_u32(&misc->bar_pfull[b]), 128);
         }
-        for (int b = 0; b < 2; ++b)
-            mbar_init(smem_u32(&misc->bar_odone[b]), 1);
+        mbar_init(smem_u32(&misc->bar_odone), 1);
         mbar_init(smem_u32(&misc->bar_never), 1);
         misc->abort = 0;
         fence_mbar_init();
@@ -1054,10 +1206,17 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     }
     if (tid >= 64 && tid < 64 + P.n_prefills)
         misc->pre[tid - 64] = P.pre[tid - 64];
+    // Dependent order (early_start = 0): the previous launch in the stream
+    // (the previous layer) must have completed, and its writes be visible,
+    // before anything it may have written is read: this layer's q/k/v may be
+    // computed from the previous layer's output.  Its CTAs signalled this
+    // launch only when they ran out of work, so the wait is short.  Without
+    // the programmatic launch attribute this is a no-op.
+    if (!P.early_start)
+        pdl_wait();
     // Consecutive launches use the workspace sets in turn, and the launch
     // that last used this one's set has completed before this one was
-    // launched (see the end of the kernel), so work starts at once, beside
-    // the previous layer's tail.
+    // launched (see the end of the kernel), so work starts at once.
     if (tid == 0) {
         misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
         // Fault injection for the bounded waits: the chosen block waits on a
@@ -1079,53 +1238,20 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     tc_fence_after();
     const uint32_t tmem = P.has_prefill ? misc->tmem_base : 0u;
 
-    uint32_t tile_cnt = 0, item_no = 0;
-    int buf = 0;
-    for (;;) {
-        const int idx = misc->item_idx[buf];
-        if (idx >= P.n_items || misc->abort)
-            break;
-        if (tid == 0)
-            misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
-        const int4 it = P.items[idx];
-        int merge_t = -1, merge_hq = 0, merge_ns = 1, merge_f = 0;
-        if ((it.x & 0xF) == ITEM_PREFILL) {
-            const int f = (int)((uint32_t)it.x >> 4);
-            const PrefillInfo &pf = misc->pre[f];
-            const int t = it.y & 0xFFFF, hq = it.y >> 16;
-            const int s = it.z & 0xFFFF, ns = it.z >> 16;
-            const int nT = (pf.chunk_start + kTileN - 1) / kTileN + t + 1;
-            const int kt0 = (int)((long long)s * nT / ns), kt1 = (int)((long long)(s + 1) * nT / ns);
-            prefill_item(P, smem, misc, tmem, pf, t, hq, kt0, kt1, ns > 1 ? it.w + s : -1, tile_cnt,
-                         item_no);
-            tile_cnt += kt1 - kt0;
-            item_no += 1;
-            if (ns > 1) {
-                merge_t = t;
-                merge_hq = hq;
-                merge_ns = ns;
-                merge_f = f;
-            }
-        } else if ((it.x & 0xF) == ITEM_DECODE_SHORT) {
-            decode_short_item(P, smem, it.y, (int)(((uint32_t)it.x >> 4) & 0x7Fu), it.z, it.w);
-        } else {
-            const uint32_t dx = (uint32_t)it.x;
-            decode_item(P, smem, misc, it.y, (int)((dx >> 4) & 0x7Fu), (int)((dx >> 11) & 0xFFFu), it.z, it.w,
-                        (int)(dx >> 23) * 16);
-        }
-        fence_proxy_async_smem();  // generic smem accesses before later TMA writes
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-        if (merge_t >= 0 && !misc->abort)
-            prefill_merge(P, misc, misc->pre[merge_f], merge_t, merge_hq, merge_ns, it.w);
-        buf ^= 1;
+    if (warp < kProdThreads / 32) {
+        regs_dec<kProdRegs>();
+        producer_loop(P, smem, misc, tmem);
+    } else {
+        regs_inc<kConsRegs>();
+        consumer_loop(P, smem, misc, tmem);
     }
+    // Every role left its loop at the same item boundary.
 
     // Out of work: wait until the previous launch has completed before
-    // exiting, so that when a later launch reuses that launch's workspace
-    // set, it is complete.  Dependent layers signal the next launch only now,
-    // so it runs after this one (its launch latency hidden).
+    // exiting (independent layers: so that when a later launch reuses that
+    // launch's workspace set, it is complete; dependent layers waited at the
+    // start already).  Dependent layers signal the next launch only now, so
+    // it runs after this one, its launch latency hidden.
     pdl_wait();
     if (!P.early_start)
         pdl_launch_dependents();
@@ -1134,8 +1260,10 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         const uint64_t t0 = globaltimer_ns();
         while (globaltimer_ns() - t0 < 200000ull)
             __nanosleep(1000);
-        __syncthreads();
     }
+    tc_fence_before();
+    named_sync(kBarItem, kThreads);
+    tc_fence_after();
     if (P.has_prefill && warp == 1)
         tmem_dealloc(tmem, kTmemCols);
     if (tid == 0) {

@@ -189,14 +189,39 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
         if (!q || (reinterpret_cast<uintptr_t>(q) & 15u))
             return report(err_buf, err_len, MX_EINVAL, "a tensor pointer is null or not 16-byte aligned");
 
-    // Work list on the stack: prefill tiles (heaviest first), then decode
-    // splits (longest first); split length chosen to fit the partial slots.
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return report(err_buf, err_len, MX_ECUDA, "cudaGetDevice failed");
+    DeviceState *st = nullptr;
+    int rc = setup_device(dev, &st, err_buf, err_len);
+    if (rc)
+        return rc;
+
+    // Work list on the stack, built by the rule of the context planner:
+    // prefill tiles (heaviest first), then decode splits (longest first),
+    // each decode cut into equal page-aligned parts.  The split length is the
+    // context planner's automatic choice, doubled while the splits exceed
+    // this entry point's partial slots or work items.
     const int hkv = g->num_kv_heads, hq = g->num_q_heads;
     const int n_qt = (p + kTileM - 1) / kTileM;
-    if ((int64_t)n_qt * hq > kNaMaxItems)
-        return report(err_buf, err_len, MX_ECAPACITY, "%d prefill tiles exceed %d work items",
-                      n_qt * hq, kNaMaxItems);
-    int split = 512;
+    const int nh = rep >= 2 ? 2 : 1;        // query heads per prefill item
+    const int n_pre = n_qt * (hq / nh);     // prefill items
+    if (n_pre > kNaMaxItems)
+        return report(err_buf, err_len, MX_ECAPACITY, "%d prefill items exceed %d work items", n_pre,
+                      kNaMaxItems);
+    int64_t total_keys = 0;
+    for (int i = 0; i < nd; ++i)
+        total_keys += (int64_t)d->decode_ctx_lens[i] + 1;
+    total_keys *= hkv;
+    int split;
+    {
+        static const double kBeside[3] = {3.5, 3.0, 2.0};
+        const double per_sm = n_qt == 0 ? 1.5 : (n_qt <= 3 ? kBeside[n_qt - 1] : 1.0);
+        const int64_t target = std::max<int64_t>(1, (int64_t)(per_sm * st->num_sms));
+        int64_t sk = (total_keys + target - 1) / target;
+        sk = (sk + 127) / 128 * 128;
+        split = (int)std::min<int64_t>(std::max<int64_t>(sk, 512), kNaMaxSplitKeys);
+    }
     auto count = [&](int sk, int64_t *parts, int64_t *items) {
         *parts = 0;
         *items = 0;
@@ -210,61 +235,60 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     int64_t parts = 0, ditems = 0;
     for (;;) {
         count(split, &parts, &ditems);
-        if ((parts <= kNaPartSlots && (int64_t)n_qt * hq + ditems <= kNaMaxItems) ||
+        if ((parts <= kNaPartSlots && (int64_t)n_pre + ditems <= kNaMaxItems) ||
             split >= kNaMaxSplitKeys)
             break;
         split = std::min(split * 2, kNaMaxSplitKeys);
     }
-    if (parts > kNaPartSlots || (int64_t)n_qt * hq + ditems > kNaMaxItems)
+    if (parts > kNaPartSlots || (int64_t)n_pre + ditems > kNaMaxItems)
         return report(err_buf, err_len, MX_ECAPACITY,
                       "decode splits need %lld partial slots / %lld items (limits %d / %d)",
-                      (long long)parts, (long long)(n_qt * hq + ditems), kNaPartSlots, kNaMaxItems);
+                      (long long)parts, (long long)(n_pre + ditems), kNaPartSlots, kNaMaxItems);
 
     alignas(16) unsigned char plan[kPlanBytes];
     DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(plan);
     int4 *items = reinterpret_cast<int4 *>(plan + (size_t)kNaMaxDecodes * sizeof(DecodeInfo));
     int n = 0;
     for (int t = n_qt - 1; t >= 0; --t)
-        for (int h = 0; h < hq; ++h)
-            items[n++] = prefill_item_code(0, t, h, 0, 1, 0);
+        for (int h = 0; h < hq; h += nh)
+            items[n++] = prefill_item_code(0, t, h, nh, 0, 1, 0);
     const int n_prefill = n;
+    // keys of each decode item, for the longest-first order (stable)
+    int32_t item_keys[kNaMaxItems];
     int part = 0;
     for (int i = 0; i < nd; ++i) {
-        const int ns = (d->decode_ctx_lens[i] + 1 + split - 1) / split;
+        const int keys = d->decode_ctx_lens[i] + 1;
+        const int ns = (keys + split - 1) / split;
+        const int len = ((keys + ns - 1) / ns + kPage - 1) / kPage * kPage;   // <= split
         dec[i].seq = d->decode_seq_ids[i];
         dec[i].ctx = d->decode_ctx_lens[i];
         dec[i].n_splits = ns;
         dec[i].part_base = ns > 1 ? part : 0;
         if (ns > 1)
             part += ns * hkv;
-    }
-    // full splits first (all have `split` keys), then the last splits by size
-    for (int i = 0; i < nd; ++i) {
-        const int ns = dec[i].n_splits;
         for (int h = 0; h < hkv; ++h)
-            for (int s = 0; s < ns - 1; ++s)
-                items[n++] = decode_item_code(i, h, s, dec[i].seq, dec[i].ctx, split);
+            for (int sp = 0; sp < ns; ++sp) {
+                int4 code = decode_item_code(i, h, sp, dec[i].seq, dec[i].ctx, len);
+                if (keys <= kPage)   // at most 16 keys: the exact short path
+                    code.x = (int32_t)(((uint32_t)code.x & ~0xFu) | (uint32_t)ITEM_DECODE_SHORT);
+                item_keys[n] = std::min(len, keys - sp * len);
+                items[n++] = code;
+            }
     }
-    const int tail0 = n;
-    for (int i = 0; i < nd; ++i)
-        for (int h = 0; h < hkv; ++h)
-            items[n++] = decode_item_code(i, h, dec[i].n_splits - 1, dec[i].seq, dec[i].ctx, split);
-    std::stable_sort(items + tail0, items + n, [&](const int4 &a, const int4 &c) {
-        const int ka = dec[a.y].ctx + 1 - (dec[a.y].n_splits - 1) * split;   // .y: decode index
-        const int kc = dec[c.y].ctx + 1 - (dec[c.y].n_splits - 1) * split;
-        return ka > kc;
-    });
-    for (int x = tail0; x < n; ++x)   // at most 16 keys: the exact short path
-        if (dec[items[x].y].ctx + 1 <= kPage)
-            items[x].x = (int32_t)(((uint32_t)items[x].x & ~0xFu) | (uint32_t)ITEM_DECODE_SHORT);
+    // stable longest-first order of the decode items (insertion sort on the
+    // stack: no allocation)
+    for (int x = n_prefill + 1; x < n; ++x) {
+        const int4 code = items[x];
+        const int32_t kx = item_keys[x];
+        int y = x;
+        for (; y > n_prefill && item_keys[y - 1] < kx; --y) {
+            items[y] = items[y - 1];
+            item_keys[y] = item_keys[y - 1];
+        }
+        items[y] = code;
+        item_keys[y] = kx;
+    }
 
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess)
-        return report(err_buf, err_len, MX_ECUDA, "cudaGetDevice failed");
-    DeviceState *st = nullptr;
-    int rc = setup_device(dev, &st, err_buf, err_len);
-    if (rc)
-        return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     uint8_t *sc = st->scratch;
 

@@ -52,6 +52,10 @@ def test_null_and_geometry_checks_without_gpu(lib):
     assert lib.mx_create(ctypes.byref(h), ctypes.byref(bad), 0) == -1
     bad = mx_geom(24, 8, 128, 16, 10, 1, 4, 8, 1)         # n_rep 3 unsupported
     assert lib.mx_create(ctypes.byref(h), ctypes.byref(bad), 0) == -1
+    # with no context, mx_error_detail reports why this thread's mx_create failed
+    buf = ctypes.create_string_buffer(256)
+    assert lib.mx_error_detail(None, buf, 256) > 0
+    assert b"geometry" in buf.value
     try:
         import torch
         has_gpu = torch.cuda.is_available()
@@ -60,3 +64,4 @@ def test_null_and_geometry_checks_without_gpu(lib):
     if not has_gpu:
         good = mx_geom(16, 8, 128, 16, 10, 1, 4, 8, 1)
         assert lib.mx_create(ctypes.byref(h), ctypes.byref(good), 0) == -6   # MX_EDEVICE
+        assert lib.mx_error_detail(None, buf, 256) > 0 and b"device" in buf.value

@@ -35,6 +35,7 @@ CASES = [
     ("qwen3-8b-attn-36L-chunk-sweep", 4096, "first"),
     ("qwen3-32b-attn-64L-chunk-sweep", 0, "first"),
     ("qwen3-32b-attn-64L-chunk-sweep", 1024, "last"),
+    ("qwen3-32b-attn-64L-chunk-sweep", 8192, "last"),     # deepest items the bench times
 ]
 
 

@@ -225,7 +225,8 @@ def test_prefill_auto_pieces_long_context():
     # a short chunk deep into a long prompt: the planner splits its tiles
     case = Case(16, [2000, 40], chunk_start=6000, p_t=200, seed=8)
     res = case.run_gpu()
-    assert res["plan"]["n_prefill_items"] > 2 * 16
+    # unsplit: 2 query tiles x 8 pairs of query heads
+    assert res["plan"]["n_prefill_items"] > 2 * 8
     _ok(case.check(res))
 
 
@@ -475,4 +476,82 @@ def test_two_chunks_of_one_sequence_rejected():
                         slots=d["slots"], prefills=[(1, 10, 20), (1, 30, 5)])   # one sequence twice
     with pytest.raises(MxError, match="EINVAL"):
         ctx.mixed_attention(bad, ctx.make_bufs(d["q"], d["k"], d["v"], d["k_pool"], d["v_pool"], d["out"]))
+    ctx.close()
+
+
+def test_several_chunks_key_pieces_repeated_calls():
+    """Two prompts' short chunks deep into long prompts (positions 6200 and
+    7000), so that the tiles of chunk 0 AND of chunk 1 are split into key
+    pieces merged by log-sum-exp, beside decodes.  The per-tile arrival
+    counters of the pieces live in the context's workspace sets, which
+    consecutive launches use in turn (three sets) and each launch resets as
+    it merges: six single-layer calls and one four-layer iteration on one
+    context reuse every set at least twice, and every row of every call must
+    match the oracle (a counter left set would leave a tile unmerged)."""
+    import oracle
+    from paper_2609_38386_gb300 import Context
+    hq, ctxs, chunks = 16, [900, 40, 2500], [(6200, 100), (7000, 100)]
+    geom, lay, slots, q, k, v, kp0, vp0 = _several_chunks_case(hq, ctxs, chunks, seed=77)
+    nd = len(ctxs)
+    prefills = [(nd + f, cs, p) for f, (cs, p) in enumerate(chunks)]
+    ctx = Context(num_q_heads=hq, num_kv_heads=8, num_pages=lay.num_pages, num_seqs=lay.num_seqs,
+                  max_pages_per_seq=lay.max_pages, max_tokens=len(slots), max_decodes=nd)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda()
+    d_q, d_k, d_v, d_kp, d_vp = t(q), t(k), t(v), t(kp0), t(vp0)
+    d_pt, d_sl = torch.from_numpy(lay.page_table).cuda(), torch.from_numpy(slots).cuda()
+    desc = ctx.make_desc(decode_seq_ids=list(range(nd)), decode_ctx_lens=ctxs, page_table=d_pt,
+                         slots=d_sl, prefills=prefills)
+    kp, vp = kp0.copy(), vp0.copy()
+    want, _ = oracle.mixed_attention(q=q, k=k, v=v, k_pool=kp, v_pool=vp, page_table=lay.page_table,
+                                     slots=slots, decode_seq_ids=np.arange(nd), decode_ctx_lens=ctxs,
+                                     prefills=prefills)
+
+    def check(out, what):
+        got = harness._bf16_to_f64(out.cpu().numpy())
+        assert np.all(np.isfinite(got)), what
+        err = np.abs(got - want)
+        assert err.max() <= MAX_ABS and err.mean() <= MEAN_ABS, (what, err.max(), err.mean())
+
+    for call in range(6):
+        d_out = torch.full((len(slots), hq, 128), 0x7FC1, dtype=torch.int16, device="cuda")
+        ctx.mixed_attention(desc, ctx.make_bufs(d_q, d_k, d_v, d_kp, d_vp, d_out))
+        ctx.sync_status()
+        if call == 0:
+            # both chunks' tiles (one item per pair of query heads) were cut
+            # into key pieces
+            n_tiles = sum(-(-p // 128) for _, p in chunks) * (hq // 2)
+            assert ctx.last_plan()["n_prefill_items"] >= 2 * n_tiles, ctx.last_plan()
+        check(d_out, f"call {call}")
+    outs = [torch.full((len(slots), hq, 128), 0x7FC1, dtype=torch.int16, device="cuda") for _ in range(4)]
+    ctx.iteration(desc, [ctx.make_bufs(d_q, d_k, d_v, d_kp, d_vp, o) for o in outs])
+    for l, o in enumerate(outs):
+        check(o, f"iteration layer {l}")
+    np.testing.assert_array_equal(d_kp.cpu().numpy().view(np.uint16), kp)
+    np.testing.assert_array_equal(d_vp.cpu().numpy().view(np.uint16), vp)
+    ctx.close()
+
+
+@pytest.mark.parametrize("hq", [16, 64])
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_short_rows_chunk_start_1_to_15(hq, seed):
+    """Chunks starting at positions 1..15 of a prompt: their first rows see
+    2..16 keys, some cached (read from a page) and some the chunk's own.
+    With so few keys the bf16 rounding of one weight of P would show, so
+    these rows are computed exactly; every row of every chunk length is
+    checked against the oracle."""
+    from synth import workload as wl
+    geom = wl.Geometry(hq)
+    lay = wl.make_layout(geom, [15 + 130 + 9], seed=seed + 100)
+    ctx = None
+    for cs in range(1, 16):
+        for p in (1, 7, 40, 130):
+            case = Case(hq, [], chunk_start=cs, p_t=p, seed=1000 * seed + 10 * cs + p, layout=lay)
+            if ctx is None:
+                from paper_2609_38386_gb300 import Context
+                ctx = Context(num_q_heads=hq, num_kv_heads=8, num_pages=lay.num_pages,
+                              num_seqs=lay.num_seqs, max_pages_per_seq=lay.max_pages,
+                              max_tokens=130, max_decodes=1)
+            err = case.check(case.run_gpu(ctx=ctx))
+            assert err["finite"] and err["pools_exact"], (cs, p, err)
+            assert err["max_abs"] <= MAX_ABS and err["mean_abs"] <= MEAN_ABS, (cs, p, err)
     ctx.close()

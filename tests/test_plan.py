@@ -20,7 +20,8 @@ def _decode_items(items):
     for x, y, z, w in items.astype(np.int64):
         ux = int(x) & 0xFFFFFFFF
         if ux & 0xF == 0:
-            pre.append(dict(f=ux >> 4, t=y & 0xFFFF, hq=y >> 16, s=z & 0xFFFF, ns=z >> 16, base=int(w)))
+            pre.append(dict(f=(ux >> 4) & 0xF, heads=((ux >> 8) & 1) + 1, t=y & 0xFFFF, hq=y >> 16,
+                            s=z & 0xFFFF, ns=z >> 16, base=int(w)))
         else:
             # 1: a split; 2: a decode of at most 16 keys (exact short path)
             assert ux & 0xF in (1, 2), hex(ux)
@@ -58,13 +59,15 @@ def _check(plan, hq, ctxs, cs, p, chunks=None):
              (n_a[d["f"]] + d["t"] + 1) * d["s"] // d["ns"] for d in pre]
     assert all(a >= b for a, b in zip(tiles, tiles[1:]))
 
-    # prefill: each (chunk, tile, head) split into pieces that partition its
-    # key tiles
+    # prefill: each (chunk, tile, pair of query heads of one KV head; one head
+    # when Hq = Hkv) split into pieces that partition its key tiles
+    nh = 2 if hq // hkv >= 2 else 1
+    assert all(d["heads"] == nh and d["hq"] % nh == 0 for d in pre)
     seen = {}
     for d in pre:
         seen.setdefault((d["f"], d["t"], d["hq"]), []).append(d)
     assert set(seen) == {(f, t, h) for f, (_, p_) in enumerate(chunks)
-                         for t in range(-(-p_ // TILE)) for h in range(hq)}
+                         for t in range(-(-p_ // TILE)) for h in range(0, hq, nh)}
     bases = []
     for (f, t, h), ps in seen.items():
         cs, p = chunks[f]
@@ -82,8 +85,8 @@ def _check(plan, hq, ctxs, cs, p, chunks=None):
         for x in ps:
             cover += range(n_t * x["s"] // ns, n_t * (x["s"] + 1) // ns)
         assert sorted(cover) == list(range(n_t))
-        if ns > 1:
-            bases.append((ps[0]["base"], ps[0]["base"] + ns))
+        if ns > 1:   # head e of piece s writes partial base + e * ns + s
+            bases.append((ps[0]["base"], ps[0]["base"] + nh * ns))
     bases.sort()
     assert all(a[1] <= b[0] for a, b in zip(bases, bases[1:]))
     assert not bases or bases[-1][1] <= PRE_PART_SLOTS
@@ -133,6 +136,8 @@ CASES = [
     (16, list(range(500, 4100, 113)), 7936, 256),
     (32, [8191] * 64, 4096, 4096),
     (64, [16383] * 128, 0, 8192),
+    (8, [100, 3000], 500, 300),          # Hq = Hkv: one query head per prefill item
+    (8, [7], 6000, 100),                 # ... and its key pieces
 ]
 
 
@@ -217,10 +222,11 @@ def test_automatic_splits_and_pieces():
     assert pl["n_items"] >= 152
     # a short chunk deep into a long prompt is cut into key pieces
     pl = _plan(16, [100], 6000, 200)
-    assert pl["n_prefill_items"] > 2 * 16
-    # a chunk with enough query tiles to fill the GPU is not
+    assert pl["n_prefill_items"] > 2 * 8
+    # a chunk with enough query tiles to fill the GPU is not (16 tiles x 8
+    # pairs of heads)
     pl = _plan(16, [100], 6000, 2048)
-    assert pl["n_prefill_items"] == 16 * 16
+    assert pl["n_prefill_items"] == 16 * 8
 
 
 def test_partial_workspace_bounds_the_split_count():
