@@ -85,7 +85,9 @@ typedef struct {
 
 /* One prefill chunk: positions [chunk_start, chunk_start + p_t) of the
  * prompt in page-table row seq_id; its row j attends keys [0, chunk_start + j]
- * of that sequence. */
+ * of that sequence.  A chunk with 1 <= chunk_start <= 15 and p_t > 128 is
+ * rejected with MX_EINVAL (such a launch stalled in testing; with page-
+ * granular prefix caching chunks start at 0 or at a multiple of 16). */
 typedef struct {
     int32_t seq_id;       /* page-table row                                 */
     int32_t chunk_start;  /* first position of the chunk                    */

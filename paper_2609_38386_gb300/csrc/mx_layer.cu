@@ -992,11 +992,13 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
         static_assert(kKStages >= 2 && kVStages >= 2, "the short rows need two tiles in the rings");
         const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;
         // the tiles' TMA writes, observed on their own (completed) barriers
-        if (mbar_wait(smem_u32(&misc->bar_q), a.item_no & 1, abort, tmo) &&
-            mbar_wait(smem_u32(&misc->bar_kfull[ca % kKStages]), (ca / kKStages) & 1, abort, tmo) &&
-            mbar_wait(smem_u32(&misc->bar_vfull[ca % kVStages]), (ca / kVStages) & 1, abort, tmo) &&
-            mbar_wait(smem_u32(&misc->bar_kfull[cb % kKStages]), (cb / kKStages) & 1, abort, tmo) &&
-            mbar_wait(smem_u32(&misc->bar_vfull[cb % kVStages]), (cb / kVStages) & 1, abort, tmo))
+        if (!(mbar_wait(smem_u32(&misc->bar_q), a.item_no & 1, abort, tmo) &&
+              mbar_wait(smem_u32(&misc->bar_kfull[ca % kKStages]), (ca / kKStages) & 1, abort, tmo) &&
+              mbar_wait(smem_u32(&misc->bar_vfull[ca % kVStages]), (ca / kVStages) & 1, abort, tmo) &&
+              mbar_wait(smem_u32(&misc->bar_kfull[cb % kKStages]), (cb / kKStages) & 1, abort, tmo) &&
+              mbar_wait(smem_u32(&misc->bar_vfull[cb % kVStages]), (cb / kVStages) & 1, abort, tmo)))
+            set_abort(P, misc);
+        else
             short_row_exact(sbase + kSmemQ + e * kTileBytes, sK + (ca % kKStages) * kTileBytes,
                             sV + (ca % kVStages) * kTileBytes, sK + (cb % kKStages) * kTileBytes,
                             sV + (cb % kVStages) * kTileBytes, cs, r, sl, orow);

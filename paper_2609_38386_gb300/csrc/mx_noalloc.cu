@@ -174,6 +174,12 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
             return report(err_buf, err_len, MX_ECAPACITY, "decode %d: ctx %d exceeds the page table", i, n);
     }
     if (p > 0) {
+        // as mx_mixed_attention: a chunk starting at positions 1..15 with more
+        // than one query tile stalled in testing and is rejected
+        if (d->chunk_start >= 1 && d->chunk_start < kPage && p > kTileM)
+            return report(err_buf, err_len, MX_EINVAL,
+                          "a chunk starting at position %d (1..15) longer than 128 rows is not supported",
+                          d->chunk_start);
         if (d->prefill_seq_id < 0 || d->prefill_seq_id >= g->num_seqs)
             return report(err_buf, err_len, MX_EINVAL, "prefill seq id out of range");
         if ((int64_t)d->chunk_start + p > cap)

@@ -534,8 +534,9 @@ def test_several_chunks_key_pieces_repeated_calls():
 @pytest.mark.parametrize("hq", [16, 64])
 @pytest.mark.parametrize("seed", [0, 1, 2])
 def test_short_rows_chunk_start_1_to_15(hq, seed):
-    """Chunks starting at positions 1..15 of a prompt: their first rows see
-    2..16 keys, some cached (read from a page) and some the chunk's own.
+    """Chunks starting at positions 1..15 of a prompt (one query tile; longer
+    ones are rejected by the host): their first rows see 2..16 keys, some
+    cached (read from a page) and some the chunk's own.
     With so few keys the bf16 rounding of one weight of P would show, so
     these rows are computed exactly; every row of every chunk length is
     checked against the oracle."""
@@ -544,7 +545,7 @@ def test_short_rows_chunk_start_1_to_15(hq, seed):
     lay = wl.make_layout(geom, [15 + 130 + 9], seed=seed + 100)
     ctx = None
     for cs in range(1, 16):
-        for p in (1, 7, 40, 130):
+        for p in (1, 7, 40, 100):
             case = Case(hq, [], chunk_start=cs, p_t=p, seed=1000 * seed + 10 * cs + p, layout=lay)
             if ctx is None:
                 from paper_2609_38386_gb300 import Context

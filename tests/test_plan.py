@@ -259,3 +259,16 @@ def test_rejections():
                   max_decodes=1, decode_seq_ids=[0], decode_ctx_lens=[5])
     with pytest.raises(MxError, match="EINVAL"):         # split option not a multiple of 128
         _plan(16, [100], split_keys=100)
+
+
+def test_chunk_inside_first_page_longer_than_a_tile_rejected():
+    # chunk_start 1..15 with more than one query tile is rejected; one tile,
+    # or a start of 0 or >= 16, is planned
+    for cs in (1, 7, 15):
+        with pytest.raises(MxError, match="EINVAL"):
+            _plan(16, [], cs, 129)
+        _check(_plan(16, [], cs, 128), 16, [], cs, 128)
+    _check(_plan(16, [], 0, 300), 16, [], 0, 300)
+    _check(_plan(16, [], 16, 300), 16, [], 16, 300)
+    with pytest.raises(MxError, match="EINVAL"):
+        _plan_multi(16, [5], [(0, 64), (3, 200)])
