@@ -85,9 +85,7 @@ typedef struct {
 
 /* One prefill chunk: positions [chunk_start, chunk_start + p_t) of the
  * prompt in page-table row seq_id; its row j attends keys [0, chunk_start + j]
- * of that sequence.  A chunk with 1 <= chunk_start <= 15 and p_t > 128 is
- * rejected with MX_EINVAL (such a launch stalled in testing; with page-
- * granular prefix caching chunks start at 0 or at a multiple of 16). */
+ * of that sequence. */
 typedef struct {
     int32_t seq_id;       /* page-table row                                 */
     int32_t chunk_start;  /* first position of the chunk                    */
@@ -250,7 +248,7 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  *     decode {1 | h << 4 | s << 11 | (len / 16) << 23, decode index i,
  *       page-table row, cached tokens ctx}: split s of decode i, KV head h,
  *       keys [s len, min((s + 1) len, ctx + 1)); kind 2 instead of 1 for a
- *       decode of at most 16 keys (one split, computed exactly in fp32);
+ *       decode of at most 64 keys (one split, computed exactly in fp32);
  *   decodes  int32 [n_decodes][4]: page-table row, ctx, number of splits,
  *     first partial slot (of head 0; head h uses base + h * splits);
  *   counts   int32 [4]: n_items, prefill items, split_keys, piece_tiles.

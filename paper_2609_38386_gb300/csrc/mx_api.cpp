@@ -177,15 +177,6 @@ int fail_to(std::string *err, int code, const char *fmt, ...)
     return code;
 }
 
-// A chunk that starts inside the prompt's first page (positions 1..15) and
-// has more than one query tile made the layer launch stall on the GPU in
-// testing, for a reason not found; such chunks are rejected.  (With
-// page-granular prefix caching a chunk starts at 0 or at a multiple of 16.)
-bool unsupported_chunk(int chunk_start, int p_t)
-{
-    return chunk_start >= 1 && chunk_start < kPage && p_t > kTileM;
-}
-
 // Host validation of a descriptor against the geometry.  need_tables: the
 // device page table and slots must be given (a launch); planning alone reads
 // only the host arrays.
@@ -209,9 +200,6 @@ int validate_desc(const mx_geom &g, const mx_iter_desc *d, bool need_tables, std
         if (x.p_t <= 0 || x.chunk_start < 0)
             return fail_to(err, MX_EINVAL, "prefill %d: p_t %d <= 0 or chunk_start %d < 0", f, x.p_t,
                            x.chunk_start);
-        if (unsupported_chunk(x.chunk_start, x.p_t))
-            return fail_to(err, MX_EINVAL, "prefill %d: a chunk starting at position %d (1..15) longer than 128 "
-                           "rows is not supported", f, x.chunk_start);
         if (x.seq_id < 0 || x.seq_id >= g.num_seqs)
             return fail_to(err, MX_EINVAL, "prefill %d: seq id %d outside [0, %d)", f, x.seq_id, g.num_seqs);
         if ((int64_t)x.chunk_start + x.p_t > cap)
@@ -235,9 +223,6 @@ int validate_desc(const mx_geom &g, const mx_iter_desc *d, bool need_tables, std
                            (long long)cap);
     }
     if (d->p_t > 0) {
-        if (unsupported_chunk(d->chunk_start, d->p_t))
-            return fail_to(err, MX_EINVAL, "a chunk starting at position %d (1..15) longer than 128 rows is not "
-                           "supported", d->chunk_start);
         if (d->prefill_seq_id < 0 || d->prefill_seq_id >= g.num_seqs)
             return fail_to(err, MX_EINVAL, "prefill seq id %d outside [0, %d)", d->prefill_seq_id,
                            g.num_seqs);
@@ -468,7 +453,7 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
                      [](const DItem &a, const DItem &b) { return a.keys > b.keys; });
     for (const DItem &x : ditems) {
         int4 code = decode_item_code(x.i, x.h, x.s, dec[x.i].seq, dec[x.i].ctx, x.len);
-        if (dec[x.i].ctx + 1 <= kPage)  // at most 16 keys: the exact short path
+        if (dec[x.i].ctx + 1 <= kShortKeys)  // few keys: the exact short path
             code.x = (int32_t)(((uint32_t)code.x & ~0xFu) | (uint32_t)ITEM_DECODE_SHORT);
         items[n++] = code;
     }

@@ -65,6 +65,22 @@ constexpr uint32_t kTmemO = 256;
 
 enum : int32_t { ITEM_PREFILL = 0, ITEM_DECODE = 1, ITEM_DECODE_SHORT = 2 };
 
+// Accuracy of rows with few keys.  With few keys one weight of P can
+// dominate the row, and the tensor-core paths multiply V by P rounded to
+// bf16: unless the row is normalised by the sum of the same rounded weights,
+// that weight's rounding (2^-9 relative, and the lazy rescale lets it reach
+// 2^8) times |v| up to ~4.5, plus the bf16 rounding of an output of
+// magnitude 2-4, can exceed the 1e-2 tolerance.
+//  - decodes of at most kShortKeys keys are computed exactly in fp32 on the
+//    CUDA cores (ITEM_DECODE_SHORT);
+//  - chunk rows of at most kShortRowKeys keys are recomputed exactly in fp32
+//    from the tiles in shared memory;
+//  - prefill items that hold positions below kShortKeys of a prompt sum the
+//    row's weights as rounded to bf16, so that P.V / l is a normalised
+//    average of V.
+constexpr int kShortKeys = 64;
+constexpr int kShortRowKeys = 16;
+
 // Prefill chunks of one iteration (several prompts' chunks may share it).
 constexpr int kMaxPrefills = 16;
 struct PrefillInfo {
@@ -83,8 +99,8 @@ struct PrefillInfo {
 //            heads - 1 (heads 1 or 2, one KV head); the tile's key tiles are
 //            split evenly between its n_s pieces; head e of piece s writes
 //            partial slot base + e * n_s + s.
-//   short decode (at most 16 keys, one split): the decode record with kind
-//            ITEM_DECODE_SHORT;
+//   short decode (at most kShortKeys keys, one split): the decode record
+//            with kind ITEM_DECODE_SHORT;
 //   decode:  {ITEM_DECODE | kv head << 4 | split index << 11 | split
 //             length / 16 << 23, decode index, page-table row, cached tokens}:
 //             split s of decode i covers keys [s * len, (s + 1) * len) of

@@ -84,16 +84,17 @@ __device__ __forceinline__ void set_abort(const LayerParams &P, Misc *misc)
 __device__ __forceinline__ float neg_inf() { return -__int_as_float(0x7f800000); }
 
 // ---------------------------------------------------------------------------
-// A decode of at most 16 keys (fewer than 16 cached tokens), KV head h: exact
-// fp32 attention on the CUDA cores.  With so few keys the bf16 rounding of a
-// single weight of P in the tensor-core path would show in the output.  The
-// scores go through shared memory; cached K/V rows are read from their page,
-// the new key from the k/v inputs (as in the split path), which it appends.
+// A decode of at most kShortKeys keys, KV head h: exact fp32 attention on the
+// CUDA cores (the bf16 rounding of one dominant weight of P in the
+// tensor-core path would show in the output).  The scores go through shared
+// memory; cached K/V rows are read from their pages, the new key from the k/v
+// inputs (as in the split path), which it appends.
 // ---------------------------------------------------------------------------
 __device__ void decode_short_item(const LayerParams &P, uint8_t *smem, int di, int h, int seq, int n, int tid)
 {
     const int nrep = P.n_rep, nk = n + 1;   // tid: consumer thread 0..255
-    float *ss = reinterpret_cast<float *>(smem);  // [kMaxRep][16] scores (log2 domain)
+    float *ss = reinterpret_cast<float *>(smem);   // [kMaxRep][kShortKeys] scores (log2 domain)
+    int *spid = reinterpret_cast<int *>(ss + kMaxRep * kShortKeys);   // page of each cached key's page
     if (tid < 32) {
         const int slot = P.slots[di];
         if (slot >= P.num_pages * kPage) {
@@ -108,51 +109,57 @@ __device__ void decode_short_item(const LayerParams &P, uint8_t *smem, int di, i
             else
                 reinterpret_cast<uint4 *>(P.v_pool + dst)[c] = __ldg(reinterpret_cast<const uint4 *>(P.v + src) + c);
         }
-    }
-    int pid = -1;
-    if (n > 0) {
-        pid = __ldg(P.page_table + (size_t)seq * P.max_pages);
-        if (pid < 0 || pid >= P.num_pages) {
-            if (tid == 0)
+    } else if (tid < 32 + kShortKeys / kPage) {
+        const int lp = tid - 32;   // page index of the sequence
+        int pid = -1;
+        if (lp * kPage < n) {
+            pid = __ldg(P.page_table + (size_t)seq * P.max_pages + lp);
+            if (pid < 0 || pid >= P.num_pages) {
                 flag_error(P, ERR_PAGE);
-            pid = -1;
+                pid = -1;
+            }
         }
+        spid[lp] = pid;
     }
+    cons_sync();
     const uint16_t *knew = P.k + ((size_t)di * P.hkv + h) * kHeadDim;
     const uint16_t *vnew = P.v + ((size_t)di * P.hkv + h) * kHeadDim;
-    const size_t pbase = ((size_t)(pid < 0 ? 0 : pid) * P.hkv + h) * kPage * kHeadDim;
-    if (tid < nrep * kPage) {
-        const int q = tid / kPage, k = tid % kPage;
+    for (int e = tid; e < nrep * kShortKeys; e += kConsThreads) {
+        const int q = e / kShortKeys, k = e % kShortKeys;
         float s = neg_inf();
-        if (k < nk && (k == n || pid >= 0)) {
+        const int pid = k < n ? spid[k / kPage] : -1;
+        if (q < nrep && k < nk && (k == n || pid >= 0)) {
             const uint4 *qr = reinterpret_cast<const uint4 *>(P.q + ((size_t)di * P.hq + h * nrep + q) * kHeadDim);
-            const uint4 *kr = reinterpret_cast<const uint4 *>(k < n ? P.k_pool + pbase + (size_t)k * kHeadDim : knew);
+            const uint4 *kr = reinterpret_cast<const uint4 *>(
+                k < n ? P.k_pool + (((size_t)pid * P.hkv + h) * kPage + k % kPage) * kHeadDim : knew);
             float acc = 0.f;
 #pragma unroll 4
             for (int c = 0; c < 16; ++c) {
                 const uint4 a = __ldg(qr + c), b = __ldg(kr + c);
                 const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    acc += bf16lo(aw[e]) * bf16lo(bw[e]) + bf16hi(aw[e]) * bf16hi(bw[e]);
+                for (int x = 0; x < 4; ++x)
+                    acc += bf16lo(aw[x]) * bf16lo(bw[x]) + bf16hi(aw[x]) * bf16hi(bw[x]);
             }
             s = acc * P.scale_log2;
         }
-        ss[q * kPage + k] = s;
+        ss[q * kShortKeys + k] = s;
     }
     cons_sync();
     for (int e = tid; e < nrep * kHeadDim; e += kConsThreads) {
         const int q = e / kHeadDim, d = e % kHeadDim;
         float m = neg_inf();
         for (int k = 0; k < nk; ++k)
-            m = fmaxf(m, ss[q * kPage + k]);
+            m = fmaxf(m, ss[q * kShortKeys + k]);
         float l = 0.f, o = 0.f;
         for (int k = 0; k < nk; ++k) {
-            const float sk = ss[q * kPage + k];
+            const float sk = ss[q * kShortKeys + k];
             if (sk == neg_inf())
                 continue;
             const float pk = ex2(sk - m);
-            const uint16_t vb = k < n ? P.v_pool[pbase + (size_t)k * kHeadDim + d] : vnew[d];
+            const int pid = k < n ? spid[k / kPage] : -1;
+            const uint16_t vb =
+                k < n ? P.v_pool[(((size_t)pid * P.hkv + h) * kPage + k % kPage) * kHeadDim + d] : vnew[d];
             l += pk;
             o += pk * __uint_as_float((uint32_t)vb << 16);
         }
@@ -508,7 +515,10 @@ __device__ __forceinline__ float row_max(const uint32_t (&sv)[128])
 }
 
 // p = 2^(s*scale - m) of one S row as bf16 pairs into TMEM at taddr (64
-// columns), and the row sum of p in 4 packed pair chains.
+// columns, stored 16 at a time), and the row sum of p in 4 packed pair
+// chains: of p as computed, or (kRoundedSum) of p as rounded to bf16, the
+// weights P.V actually uses.
+template <bool kRoundedSum>
 __device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float sl, float nm, uint32_t taddr)
 {
     float rs8[8];
@@ -516,18 +526,21 @@ __device__ __forceinline__ float row_exp_store(const uint32_t (&sv)[128], float 
     for (int u = 0; u < 8; ++u)
         rs8[u] = 0.f;
 #pragma unroll
-    for (int half = 0; half < 2; ++half) {
-        uint32_t pk[32];
+    for (int q = 0; q < 4; ++q) {
+        uint32_t pk[16];
 #pragma unroll
-        for (int cc = 0; cc < 32; ++cc) {
-            const int k0 = 64 * half + 2 * cc;
+        for (int cc = 0; cc < 16; ++cc) {
+            const int k0 = 32 * q + 2 * cc;
             float x0, x1;
             ffma2(x0, x1, __uint_as_float(sv[k0]), __uint_as_float(sv[k0 + 1]), sl, sl, nm, nm);
             const float e0 = ex2(x0), e1 = ex2(x1);
-            fadd2(rs8[2 * (cc & 3)], rs8[2 * (cc & 3) + 1], e0, e1);
             pk[cc] = pack_bf16(e0, e1);
+            if (kRoundedSum)
+                fadd2(rs8[2 * (cc & 3)], rs8[2 * (cc & 3) + 1], bf16lo(pk[cc]), bf16hi(pk[cc]));
+            else
+                fadd2(rs8[2 * (cc & 3)], rs8[2 * (cc & 3) + 1], e0, e1);
         }
-        tmem_st32(taddr + 32 * half, pk);
+        tmem_st16(taddr + 16 * q, pk);
     }
     return ((rs8[0] + rs8[1]) + (rs8[2] + rs8[3])) + ((rs8[4] + rs8[5]) + (rs8[6] + rs8[7]));
 }
@@ -542,26 +555,27 @@ __device__ __forceinline__ uint4 sw128_chunk(uint32_t base, int row, int c)
     return v;
 }
 
-// Chunk row r of a chunk that starts at position cs, with cs + r < 16,
-// attends only keys 0..cs+r.  With so few keys the bf16 rounding of a single
-// weight of P would show in the output, so such a row is recomputed here in
-// fp32 from the tiles still in shared memory and its output row overwritten:
-// key k < cs is row k of the cached tile (sKa, sVa: the item's first key
-// tile), key k >= cs is row k - cs of the chunk's own first tile (sKb, sVb).
+// Chunk row r of a chunk that starts at position cs, with cs + r <
+// kShortRowKeys, attends only keys 0..cs+r.  With so few keys the bf16 rounding
+// of a dominant weight of P would show in the output, so such a row is
+// recomputed here in fp32 from the tiles still in shared memory and its
+// output row overwritten: key k < cs is row k of the cached tile (sKa, sVa:
+// the item's first key tile), key k >= cs is row k - cs of the chunk's own
+// first tile (sKb, sVb).
 __device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKa, uint32_t sVa, uint32_t sKb,
                                                 uint32_t sVb, int cs, int r, float sl, uint16_t *orow)
 {
-    const int last = cs + r;   // keys 0..last, last < 16
-    float s[16];
+    const int last = cs + r;   // keys 0..last, last < kShortRowKeys
+    float s[kShortRowKeys];
 #pragma unroll
-    for (int k = 0; k < 16; ++k)
+    for (int k = 0; k < kShortRowKeys; ++k)
         s[k] = 0.f;
 #pragma unroll 1
     for (int c = 0; c < 16; ++c) {
         const uint4 q4 = sw128_chunk(sQ, r, c);
         const uint32_t qw[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
+        for (int k = 0; k < kShortRowKeys; ++k) {
             if (k <= last) {
                 const uint4 k4 = k < cs ? sw128_chunk(sKa, k, c) : sw128_chunk(sKb, k - cs, c);
                 const uint32_t kw[4] = {k4.x, k4.y, k4.z, k4.w};
@@ -573,12 +587,12 @@ __device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKa, uint3
     }
     float m = neg_inf();
 #pragma unroll
-    for (int k = 0; k < 16; ++k)
+    for (int k = 0; k < kShortRowKeys; ++k)
         if (k <= last)
             m = fmaxf(m, s[k] * sl);
     float l = 0.f;
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
+    for (int k = 0; k < kShortRowKeys; ++k) {
         s[k] = k <= last ? ex2(s[k] * sl - m) : 0.f;
         l += s[k];
     }
@@ -590,7 +604,7 @@ __device__ __forceinline__ void short_row_exact(uint32_t sQ, uint32_t sKa, uint3
         for (int e = 0; e < 8; ++e)
             acc[e] = 0.f;
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
+        for (int k = 0; k < kShortRowKeys; ++k) {
             if (k <= last) {
                 const uint4 v4 = k < cs ? sw128_chunk(sVa, k, c) : sw128_chunk(sVb, k - cs, c);
                 const uint32_t vw[4] = {v4.x, v4.y, v4.z, v4.w};
@@ -883,10 +897,15 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
     volatile int *abort = &misc->abort;
     const uint64_t tmo = P.timeout_ns;
 
+    // the item holds a prompt's first positions, where a row has few keys
+    const bool few_keys = a.t == 0 && cs < kShortKeys;
     float m_run = neg_inf(), l_run = 0.f;
     bool ok = true;
     for (int i = 0; i < nT; ++i) {
-        if (!mbar_wait(smem_u32(&misc->bar_sfull[e]), (ph0 + i) & 1, abort, tmo)) {
+        // the warp agrees on the outcome: the TMEM accesses below are
+        // warp-collective, so no lane may leave the loop alone
+        const bool got = mbar_wait(smem_u32(&misc->bar_sfull[e]), (ph0 + i) & 1, abort, tmo);
+        if (!__all_sync(0xffffffffu, got)) {
             ok = false;
             break;
         }
@@ -911,13 +930,16 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
         const bool rescale = m_new > m_run + 8.0f;
         const float m_use = rescale ? m_new : m_run;
         // P over the first 64 columns of S (the A operand of P.V)
-        const float rs = row_exp_store(sv, sl, -m_use, tS);
+        const float rs = few_keys ? row_exp_store<true>(sv, sl, -m_use, tS) : row_exp_store<false>(sv, sl, -m_use, tS);
         // FA4-style lazy rescale: O moves only when the row max grows by more
         // than 8 in log2 units.  O_e is stable here: sfull of this tile was
         // committed after O_e += P_e V of the previous tile, and the next P.V
-        // waits for this tile's P.
-        if (rescale && i > 0) {
-            const float alpha = ex2(m_run - m_use);
+        // waits for this tile's P.  tcgen05.ld/st are warp-collective, so the
+        // whole warp rescales when any of its rows must (alpha = 1 for the
+        // others): a branch taken by some lanes only would run them in a
+        // diverged warp.
+        if (i > 0 && __any_sync(0xffffffffu, rescale)) {
+            const float alpha = rescale ? ex2(m_run - m_use) : 1.0f;
 #pragma unroll
             for (int gq = 0; gq < 4; ++gq) {
                 uint32_t o[32];
@@ -938,7 +960,7 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
     }
     if (ok && !mbar_wait(smem_u32(&misc->bar_odone), a.item_no & 1, abort, tmo))
         ok = false;
-    if (!ok) {
+    if (!__all_sync(0xffffffffu, ok)) {   // warp-uniform, as above
         set_abort(P, misc);
         return;
     }
@@ -983,11 +1005,12 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
             }
         }
     }
-    // rows with at most 16 keys (positions 0..15 of a prompt): exact fp32
-    // recomputation.  The item (t = 0, never split) has one key tile (cs = 0)
-    // or two (0 < cs < 16: the cached tile, then the chunk's own), all still
-    // in their K and V stages (at least two of each).
-    if (a.t == 0 && cs < kPage && cs + r < kPage && j < p) {
+    // rows with at most kShortRowKeys keys (positions 0..15 of a prompt):
+    // exact fp32 recomputation.  The item (t = 0, never split) has one key
+    // tile (cs = 0) or two (0 < cs < 16: the cached tile, then the chunk's
+    // own), all still in their K and V stages (at least two of each).
+    static_assert(kShortRowKeys <= kTileN, "the short rows' keys lie in the first two tiles");
+    if (a.t == 0 && cs < kShortRowKeys && cs + r < kShortRowKeys && j < p) {
         const uint32_t ca = a.tile0, cb = a.tile0 + (cs > 0 ? 1u : 0u);
         static_assert(kKStages >= 2 && kVStages >= 2, "the short rows need two tiles in the rings");
         const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;

@@ -174,12 +174,6 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
             return report(err_buf, err_len, MX_ECAPACITY, "decode %d: ctx %d exceeds the page table", i, n);
     }
     if (p > 0) {
-        // as mx_mixed_attention: a chunk starting at positions 1..15 with more
-        // than one query tile stalled in testing and is rejected
-        if (d->chunk_start >= 1 && d->chunk_start < kPage && p > kTileM)
-            return report(err_buf, err_len, MX_EINVAL,
-                          "a chunk starting at position %d (1..15) longer than 128 rows is not supported",
-                          d->chunk_start);
         if (d->prefill_seq_id < 0 || d->prefill_seq_id >= g->num_seqs)
             return report(err_buf, err_len, MX_EINVAL, "prefill seq id out of range");
         if ((int64_t)d->chunk_start + p > cap)
@@ -275,7 +269,7 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
         for (int h = 0; h < hkv; ++h)
             for (int sp = 0; sp < ns; ++sp) {
                 int4 code = decode_item_code(i, h, sp, dec[i].seq, dec[i].ctx, len);
-                if (keys <= kPage)   // at most 16 keys: the exact short path
+                if (keys <= kShortKeys)   // few keys: the exact short path
                     code.x = (int32_t)(((uint32_t)code.x & ~0xFu) | (uint32_t)ITEM_DECODE_SHORT);
                 item_keys[n] = std::min(len, keys - sp * len);
                 items[n++] = code;

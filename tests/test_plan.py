@@ -10,6 +10,7 @@ import pytest
 from paper_2609_38386_gb300 import MxError, plan_work
 
 PAGE, TILE = 16, 128
+SHORT_KEYS = 64             # rows of at most this many keys take the exact path
 PART_SLOTS = 16384          # decode split partials of a context
 PRE_PART_SLOTS = 1024       # prefill piece partials of a context
 
@@ -23,9 +24,9 @@ def _decode_items(items):
             pre.append(dict(f=(ux >> 4) & 0xF, heads=((ux >> 8) & 1) + 1, t=y & 0xFFFF, hq=y >> 16,
                             s=z & 0xFFFF, ns=z >> 16, base=int(w)))
         else:
-            # 1: a split; 2: a decode of at most 16 keys (exact short path)
+            # 1: a split; 2: a decode of at most 64 keys (exact short path)
             assert ux & 0xF in (1, 2), hex(ux)
-            assert ux & 0xF == 1 or int(w) + 1 <= PAGE
+            assert ux & 0xF == 1 or int(w) + 1 <= SHORT_KEYS
             dec.append(dict(kind=ux & 0xF, h=(ux >> 4) & 0x7F, s=(ux >> 11) & 0xFFF, len=(ux >> 23) * 16,
                             i=int(y), row=int(z), ctx=int(w)))
     return pre, dec
@@ -51,9 +52,10 @@ def _check(plan, hq, ctxs, cs, p, chunks=None):
     pre, dec = _decode_items(items)
     assert len(pre) == plan["n_prefill_items"]
     # claim order: every prefill item first, heaviest first; then decode
-    # splits, longest first
+    # splits (and exact short decodes), longest first
     kinds = [(int(x) & 0xF) for x in items[:, 0]]
-    assert kinds == sorted(kinds)
+    n_pre = kinds.count(0)
+    assert kinds[:n_pre] == [0] * n_pre
     n_a = [-(-c // TILE) for c, _ in chunks]
     tiles = [(n_a[d["f"]] + d["t"] + 1) * (d["s"] + 1) // d["ns"] -
              (n_a[d["f"]] + d["t"] + 1) * d["s"] // d["ns"] for d in pre]
@@ -99,7 +101,7 @@ def _check(plan, hq, ctxs, cs, p, chunks=None):
     seen = {}
     for d in dec:
         assert d["row"] == d["i"] and d["ctx"] == ctxs[d["i"]]
-        assert d["kind"] == (2 if ctxs[d["i"]] + 1 <= PAGE else 1)   # the exact short path
+        assert d["kind"] == (2 if ctxs[d["i"]] + 1 <= SHORT_KEYS else 1)   # the exact short path
         assert d["len"] % PAGE == 0 and 0 < d["len"] <= 4096
         seen.setdefault((d["i"], d["h"]), []).append(d)
     assert set(seen) == {(i, h) for i in range(len(ctxs)) for h in range(hkv)}
@@ -260,15 +262,3 @@ def test_rejections():
     with pytest.raises(MxError, match="EINVAL"):         # split option not a multiple of 128
         _plan(16, [100], split_keys=100)
 
-
-def test_chunk_inside_first_page_longer_than_a_tile_rejected():
-    # chunk_start 1..15 with more than one query tile is rejected; one tile,
-    # or a start of 0 or >= 16, is planned
-    for cs in (1, 7, 15):
-        with pytest.raises(MxError, match="EINVAL"):
-            _plan(16, [], cs, 129)
-        _check(_plan(16, [], cs, 128), 16, [], cs, 128)
-    _check(_plan(16, [], 0, 300), 16, [], 0, 300)
-    _check(_plan(16, [], 16, 300), 16, [], 16, 300)
-    with pytest.raises(MxError, match="EINVAL"):
-        _plan_multi(16, [5], [(0, 64), (3, 200)])
