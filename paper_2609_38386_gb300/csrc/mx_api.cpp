@@ -42,7 +42,7 @@ constexpr int kPartSlots = 16384;     // decode split partials capacity
 // launch n has completed and its set is free again.
 constexpr int kWorkSets = 3;
 constexpr int kPrePartSlots = 1024;   // prefill piece partials capacity (64 KiB each)
-constexpr int kMinPieceTiles = 48;    // smallest prefill piece, in 128-key tiles
+constexpr int kMinPieceTiles = 16;    // smallest prefill piece, in 128-key tiles
 constexpr int kMaxSplitKeys = kWarps * 32 * kPage;  // 4096: one page id per lane
 constexpr uint64_t kTimeoutNs = 1000000000ull;      // 1 s bound on in-kernel waits
 
@@ -371,14 +371,17 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
             pre_work += (int64_t)(nA + t + 1) * n_grp;
     }
     // Splitting costs a partial write and a merge; it pays only when the
-    // chunk has too few tiles to occupy the GPU (short chunks deep into a
-    // long prompt), so tiles are split only then, into >= 48-tile pieces.
+    // chunk has too few items to occupy the GPU (short chunks deep into a
+    // long prompt), so tiles are split only then, into pieces of twice the
+    // per-SM share of the prefill work, at least 16 tiles (on the 0.6B
+    // sweep's 256- to 1024-row chunks at position 4096 this matched the best
+    // of a 8-32-tile sweep; wider geometries have enough items unsplit).
     int piece = k.piece_tiles_opt;
     if (piece <= 0) {
         if ((int64_t)n_qt * n_grp * 2 >= k.num_sms)
             piece = 65535;
         else
-            piece = (int)std::max<int64_t>(kMinPieceTiles, (pre_work + k.num_sms - 1) / k.num_sms);
+            piece = (int)std::max<int64_t>(kMinPieceTiles, 2 * ((pre_work + k.num_sms - 1) / k.num_sms));
     }
     auto count_pre_parts = [&](int pc) {
         int64_t parts = 0;

@@ -91,27 +91,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
     }
 }
 
-// The same bound, polling with the non-blocking test_wait only: a thread
-// suspended in try_wait resumes some hundred cycles after the phase
-// completes, which the MMA-issuing thread pays between MMA groups.
-__device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity,
-                                               volatile int *abort, uint64_t limit_ns)
-{
-    if (mbar_test_wait(bar, parity))
-        return true;
-    const uint64_t t0 = globaltimer_ns();
-    for (uint32_t it = 1;; ++it) {
-        if (mbar_test_wait(bar, parity))
-            return true;
-        if ((it & 255u) == 0) {
-            if (*abort)
-                return false;
-            if (globaltimer_ns() - t0 > limit_ns)
-                return false;
-        }
-    }
-}
-
 // Programmatic dependent launch: allow the next kernel in the stream to be
 // launched, and wait until the previous kernel has completed and its memory
 // operations are visible (both no-ops without the launch attribute).
