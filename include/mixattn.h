@@ -214,6 +214,13 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
  * reported error the context clears its counters and stays usable. */
 #define MX_OPT_WAIT_LIMIT_US 5
 #define MX_OPT_TEST_STALL_BLOCK 6
+/* MX_OPT_V_STAGES: depth of the value-tile ring of prefill items, 2 or 3
+ * (0 = automatic: 3 when the launch's prefill tensor work in flops is at
+ * least 150 times its decode key/value bytes, else 2).  Three stages hide
+ * the value loads of long prefill items but take 224 KiB of shared memory
+ * per SM instead of 192, and the smaller L1 slows decode-heavy launches.
+ * Results are the same either way. */
+#define MX_OPT_V_STAGES 7
 int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 
 /* Number of work items and decode split length chosen for the last planned

@@ -88,6 +88,7 @@ struct mx_ctx {
     int pdl = 1;  // MX_OPT_PDL: 0 stream order, 1 dependent layers, 2 independent layers
     uint64_t wait_limit_ns = kTimeoutNs;  // MX_OPT_WAIT_LIMIT_US
     int stall_block = -1;                 // MX_OPT_TEST_STALL_BLOCK - 1
+    int v_stages_opt = 0;                 // MX_OPT_V_STAGES (0 = automatic)
     size_t merge_bytes = 0, pre_cnt_bytes = 0;
     // last plan
     int last_items = 0, last_split = 0, last_prefill_items = 0, last_piece_tiles = 0;
@@ -137,6 +138,7 @@ struct Plan {
     int n_items = 0;
     int n_prefill = 0;
     int split_keys = 0;
+    int v_stages = 2;
     int slot = 0;
     const int4 *items_dev = nullptr;
     const DecodeInfo *dec_dev = nullptr;
@@ -299,9 +301,10 @@ struct PlanKnobs {
     int piece_tiles_opt;   // 0 = automatic
     int pdl;               // launch order (MX_OPT_PDL)
     int max_items;         // capacity of the items array
+    int v_stages_opt = 0;  // MX_OPT_V_STAGES (0 = automatic)
 };
 struct WorkList {
-    int n_items = 0, n_prefill = 0, n_prefills = 0, split_keys = 0, piece_tiles = 0;
+    int n_items = 0, n_prefill = 0, n_prefills = 0, split_keys = 0, piece_tiles = 0, v_stages = 2;
 };
 
 // a1: the per-iteration work list, on the host, into dec[n_decodes] and
@@ -461,11 +464,19 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
         items[n++] = code;
     }
 
+    // V ring depth: the prefill chunks' causal tensor work against the
+    // decode splits' key/value bytes
+    double pre_flops = 0.0;
+    for (const PrefillInfo &x : pfs)
+        pre_flops += 4.0 * hq * kHeadDim * ((double)x.p_t * x.chunk_start + 0.5 * (double)x.p_t * (x.p_t + 1));
+    const double dec_bytes = (double)total_keys * kHeadDim * 2 * 2;
+
     out->n_items = n;
     out->n_prefill = n_prefill;
     out->n_prefills = n_pf;
     out->split_keys = split;
     out->piece_tiles = piece;
+    out->v_stages = k.v_stages_opt > 0 ? k.v_stages_opt : choose_v_stages(pre_flops, dec_bytes);
     return MX_OK;
 }
 
@@ -486,7 +497,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     PrefillInfo *pre = reinterpret_cast<PrefillInfo *>(host + pre_off);
     const size_t items_off = pre_off + (size_t)kMaxPrefills * sizeof(PrefillInfo);
     int4 *items = reinterpret_cast<int4 *>(host + items_off);
-    const PlanKnobs knobs{c->num_sms, c->split_keys_opt, c->piece_tiles_opt, c->pdl, c->max_items};
+    const PlanKnobs knobs{c->num_sms, c->split_keys_opt, c->piece_tiles_opt, c->pdl, c->max_items, c->v_stages_opt};
     WorkList wl;
     int rc = build_work_list(c->g, d, knobs, dec, pre, items, &wl, &c->last_error);
     if (rc)
@@ -515,6 +526,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     out->n_items = n;
     out->n_prefill = wl.n_prefill;
     out->split_keys = wl.split_keys;
+    out->v_stages = wl.v_stages;
     out->slot = slot;
     out->items_dev = reinterpret_cast<const int4 *>(c->plan_dev[slot] + items_off);
     out->dec_dev = reinterpret_cast<const DecodeInfo *>(c->plan_dev[slot]);
@@ -576,6 +588,7 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->max_pages = g.max_pages_per_seq;
     P->split_keys = pl.split_keys;
     P->has_prefill = pl.n_prefill > 0 ? 1 : 0;
+    P->v_stages = pl.v_stages;
     P->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     P->timeout_ns = c->wait_limit_ns;
     P->stall_block = c->stall_block;
@@ -982,6 +995,11 @@ int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
         if (value < 0 || value > 65535)
             return fail(c, MX_EINVAL, "stall block must be in [0, 65535]");
         c->stall_block = (int)value - 1;
+        return MX_OK;
+    case MX_OPT_V_STAGES:
+        if (value != 0 && value != 2 && value != 3)
+            return fail(c, MX_EINVAL, "MX_OPT_V_STAGES is 0, 2 or 3");
+        c->v_stages_opt = (int)value;
         return MX_OK;
     default:
         return fail(c, MX_EINVAL, "unknown option %d", option);

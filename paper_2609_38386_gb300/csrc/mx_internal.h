@@ -35,24 +35,42 @@ constexpr int kHalfTile = kTileM * 64 * 2;             // 128 rows x 64 bf16 = 1
 constexpr int kTileBytes = 2 * kHalfTile;              // 32 KiB
 // A prefill item serves one or two query heads of one KV head: a Q tile per
 // head, and K / V rings shared by both.  K stage c % kKStages is released
-// once both heads' S_c = Q K_c^T have completed, V stage c % kVStages once
-// both heads' P_c V_c have.
+// once both heads' S_c = Q K_c^T have completed, V stage c % v_stages once
+// both heads' P_c V_c have.  A V tile can be requested only when the P.V two
+// (or three) tiles back has completed, one tile period before (or two before)
+// its own P.V, and under load a tile takes about as long as a period to land:
+// launches with a large prefill share use three V stages (224 KiB of shared
+// memory); the others use two, which leaves 32 KiB more to the L1 cache that
+// the decode splits and short items depend on.
 constexpr int kKStages = 2;
-constexpr int kVStages = 2;
+constexpr int kVStagesMax = 3;
 constexpr int kSmemQ = 0;                              // Q of head 0, then head 1
 constexpr int kSmemK = kSmemQ + 2 * kTileBytes;
 constexpr int kSmemV = kSmemK + kKStages * kTileBytes;
-constexpr int kSmemData = kSmemV + kVStages * kTileBytes;   // 192 KiB
-constexpr int kSmemMisc = kSmemData;                   // barriers etc.
 constexpr int kSmemMiscBytes = 1024;
-constexpr int kSmemTotal = kSmemData + kSmemMiscBytes + 1024;  // + alignment slack
+// Data (192 or 224 KiB), then the barrier block at its end.
+__host__ __device__ constexpr int smem_data_bytes(int v_stages) { return kSmemV + v_stages * kTileBytes; }
+__host__ __device__ constexpr int smem_total_bytes(int v_stages)
+{
+    return smem_data_bytes(v_stages) + kSmemMiscBytes + 1024;   // + alignment slack
+}
+constexpr int kSmemTotalMax = smem_total_bytes(kVStagesMax);
+static_assert(kSmemTotalMax <= 227 * 1024, "shared memory per CTA");
+
+// Launch rule for the V ring depth: three stages when the launch's prefill
+// tensor work (flops) is at least 150 times its decode key/value bytes (at
+// the measured peaks, about 0.65 of the decode streaming time).
+__host__ __device__ inline int choose_v_stages(double prefill_flops, double decode_bytes)
+{
+    return prefill_flops > 0.0 && prefill_flops >= 150.0 * decode_bytes ? 3 : 2;
+}
 
 // Decode ring: each of the 8 decode warps owns kDecStages stages of one page
 // (K 4 KiB + V 4 KiB).
 constexpr int kPageBytes = kPage * kHeadDim * 2;       // 4 KiB
 constexpr int kDecStageBytes = 2 * kPageBytes;         // 8 KiB
 constexpr int kDecStages = 3;
-static_assert(kWarps * kDecStages * kDecStageBytes <= kSmemData, "decode ring too large");
+static_assert(kWarps * kDecStages * kDecStageBytes <= smem_data_bytes(2), "decode ring too large");
 
 // TMEM columns (fp32): S of head 0 [0,128), S of head 1 [128,256), O of
 // head 0 [256,384), O of head 1 [384,512).  P_h (bf16 pairs, the A operand
@@ -171,6 +189,7 @@ struct LayerParams {
     int32_t num_pages, max_pages;
     int32_t split_keys;    // keys per decode split (multiple of 128)
     int32_t has_prefill;   // allocate TMEM only when prefill tiles exist
+    int32_t v_stages;      // V ring depth of prefill items (2 or 3); sets the shared memory size
     int32_t early_start;   // let the next launch start as soon as this one is resident
     float scale_log2;      // log2(e) / sqrt(head_dim)
     uint64_t timeout_ns;   // bound on every in-kernel wait

@@ -46,8 +46,8 @@ struct Misc {
     uint64_t bar_q;                   // Q tiles of the item landed
     uint64_t bar_kfull[kKStages];     // K tile landed
     uint64_t bar_kempty[kKStages];    // both heads' S = Q K^T of that tile done
-    uint64_t bar_vfull[kVStages];     // V tile landed
-    uint64_t bar_vempty[kVStages];    // both heads' P V of that tile done
+    uint64_t bar_vfull[kVStagesMax];  // V tile landed
+    uint64_t bar_vempty[kVStagesMax]; // both heads' P V of that tile done
     uint64_t bar_sfull[2];            // S_h ready for head h's softmax
     uint64_t bar_pfull[2];            // P_h written by head h's 128 softmax threads
     uint64_t bar_odone;               // every MMA of the item done
@@ -673,7 +673,7 @@ __device__ void prefill_load_ring(const LayerParams &P, Misc *misc, const Prefil
     const int cs = pf.chunk_start, tb = pf.token_base;
     const int nA = (cs + kTileN - 1) / kTileN;
     const int nT = a.kt1 - a.kt0;
-    const int nst = isK ? kKStages : kVStages;
+    const int nst = isK ? kKStages : P.v_stages;
     const void *tm_pool = isK ? (const void *)&P.tm_kpool : (const void *)&P.tm_vpool;
     const void *tm_in = isK ? (const void *)&P.tm_k : (const void *)&P.tm_v;
     uint64_t *full = isK ? misc->bar_kfull : misc->bar_vfull;
@@ -696,10 +696,10 @@ __device__ void prefill_load_ring(const LayerParams &P, Misc *misc, const Prefil
         return pid;
     };
     int pid_cur = fetch_pids(0), pid_next = fetch_pids(4);
-    for (int i = 0; i < nT; ++i) {
-        const uint32_t c = a.tile0 + i;
-        const int st = c % nst;
-        const uint32_t ph = (c / nst) & 1;
+    // ring stage and phase of tile a.tile0 + i, advanced without a division
+    int st = (int)(a.tile0 % (uint32_t)nst);
+    uint32_t ph = (a.tile0 / (uint32_t)nst) & 1;
+    for (int i = 0; i < nT; ++i, st = st + 1 == nst ? 0 : st + 1, ph ^= st == 0 ? 1u : 0u) {
         const int gi = a.kt0 + i;
         if (i > 0 && (i & 3) == 0) {
             pid_cur = pid_next;
@@ -756,6 +756,10 @@ __device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs 
     volatile int *abort = &misc->abort;
     const uint64_t tmo = P.timeout_ns;
     const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;
+    const uint32_t vst = (uint32_t)P.v_stages;
+    // V stage and phase of the tile whose P.V comes next, advanced without a
+    // division (the ring depth is a launch parameter)
+    uint32_t vs = a.tile0 % vst, vph = (a.tile0 / vst) & 1;
     bool ok = mbar_wait(smem_u32(&misc->bar_q), a.item_no & 1, abort, tmo);
     tc_fence_after();
     const uint64_t qd0 = smem_desc(sbase + kSmemQ, 16, 1024, kSwz128);
@@ -763,13 +767,13 @@ __device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs 
     for (int j = 0; ok && j <= nT; ++j) {
         const uint32_t c = a.tile0 + j;
         uint64_t vdesc = 0;
+        const uint32_t vs_cur = vs;
         if (j > 0) {
-            const uint32_t cp = c - 1;
-            if (!mbar_wait(smem_u32(&misc->bar_vfull[cp % kVStages]), (cp / kVStages) & 1, abort, tmo)) {
+            if (!mbar_wait(smem_u32(&misc->bar_vfull[vs_cur]), vph, abort, tmo)) {
                 ok = false;
                 break;
             }
-            const uint32_t dv = sV + (cp % kVStages) * kTileBytes;
+            const uint32_t dv = sV + vs_cur * kTileBytes;
             if (a.kt0 + j - 1 == nA - 1 && (cs % kTileN) != 0)
                 clear_uncached_rows(dv, cs - (a.kt0 + j - 1) * kTileN);
             vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
@@ -824,8 +828,11 @@ __device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs 
             break;
         if (j < nT)
             tc_commit(smem_u32(&misc->bar_kempty[c % kKStages]));
-        if (j > 0)
-            tc_commit(smem_u32(&misc->bar_vempty[(c - 1) % kVStages]));
+        if (j > 0) {
+            tc_commit(smem_u32(&misc->bar_vempty[vs_cur]));
+            vs = vs + 1 == vst ? 0u : vs + 1;
+            vph ^= vs == 0 ? 1u : 0u;
+        }
     }
     if (ok)
         tc_commit(smem_u32(&misc->bar_odone));
@@ -1012,19 +1019,20 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
     static_assert(kShortRowKeys <= kTileN, "the short rows' keys lie in the first two tiles");
     if (a.t == 0 && cs < kShortRowKeys && cs + r < kShortRowKeys && j < p) {
         const uint32_t ca = a.tile0, cb = a.tile0 + (cs > 0 ? 1u : 0u);
-        static_assert(kKStages >= 2 && kVStages >= 2, "the short rows need two tiles in the rings");
+        static_assert(kKStages >= 2, "the short rows need two tiles in the rings");   // and v_stages >= 2
         const uint32_t sK = sbase + kSmemK, sV = sbase + kSmemV;
+        const uint32_t vst = (uint32_t)P.v_stages;
         // the tiles' TMA writes, observed on their own (completed) barriers
         if (!(mbar_wait(smem_u32(&misc->bar_q), a.item_no & 1, abort, tmo) &&
               mbar_wait(smem_u32(&misc->bar_kfull[ca % kKStages]), (ca / kKStages) & 1, abort, tmo) &&
-              mbar_wait(smem_u32(&misc->bar_vfull[ca % kVStages]), (ca / kVStages) & 1, abort, tmo) &&
+              mbar_wait(smem_u32(&misc->bar_vfull[ca % vst]), (ca / vst) & 1, abort, tmo) &&
               mbar_wait(smem_u32(&misc->bar_kfull[cb % kKStages]), (cb / kKStages) & 1, abort, tmo) &&
-              mbar_wait(smem_u32(&misc->bar_vfull[cb % kVStages]), (cb / kVStages) & 1, abort, tmo)))
+              mbar_wait(smem_u32(&misc->bar_vfull[cb % vst]), (cb / vst) & 1, abort, tmo)))
             set_abort(P, misc);
         else
             short_row_exact(sbase + kSmemQ + e * kTileBytes, sK + (ca % kKStages) * kTileBytes,
-                            sV + (ca % kVStages) * kTileBytes, sK + (cb % kKStages) * kTileBytes,
-                            sV + (cb % kVStages) * kTileBytes, cs, r, sl, orow);
+                            sV + (ca % vst) * kTileBytes, sK + (cb % kKStages) * kTileBytes,
+                            sV + (cb % vst) * kTileBytes, cs, r, sl, orow);
     }
 }
 
@@ -1196,7 +1204,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    Misc *misc = reinterpret_cast<Misc *>(smem + kSmemMisc);
+    Misc *misc = reinterpret_cast<Misc *>(smem + smem_data_bytes(P.v_stages));
     const int tid = threadIdx.x, warp = tid >> 5;
 
     if (tid == 0) {
@@ -1205,7 +1213,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
             mbar_init(smem_u32(&misc->bar_kempty[b]), 1);
         }
-        for (int b = 0; b < kVStages; ++b) {
+        for (int b = 0; b < P.v_stages; ++b) {
             mbar_init(smem_u32(&misc->bar_vfull[b]), 1);
             mbar_init(smem_u32(&misc->bar_vempty[b]), 1);
         }
@@ -1335,7 +1343,7 @@ __global__ void kv_append_kernel(const int32_t *__restrict__ slots, int n_tokens
 cudaError_t init_layer_kernel()
 {
     return cudaFuncSetAttribute(mixed_layer_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kSmemTotal);
+                                kSmemTotalMax);
 }
 
 cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream, bool pdl)
@@ -1343,7 +1351,7 @@ cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stre
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemTotal;
+    cfg.dynamicSmemBytes = smem_total_bytes(P.v_stages);   // only what the launch uses: the rest is L1
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -326,6 +326,8 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     P.max_pages = g->max_pages_per_seq;
     P.split_keys = split;
     P.has_prefill = n_prefill > 0 ? 1 : 0;
+    P.v_stages = choose_v_stages(4.0 * hq * kHeadDim * ((double)p * pre.chunk_start + 0.5 * (double)p * (p + 1)),
+                                 (double)total_keys * kHeadDim * 2 * 2);
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     P.timeout_ns = 1000000000ull;
     P.stall_block = -1;

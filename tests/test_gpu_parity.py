@@ -221,6 +221,32 @@ def test_prefill_key_pieces(piece, cs, p):
     _ok(case.check(res))
 
 
+@pytest.mark.parametrize("v_stages", [2, 3])
+@pytest.mark.parametrize("hq,ctx,cs,p", [(16, [900, 3, 64], 0, 300), (64, [2000, 17], 1000, 260),
+                                         (32, [], 77, 700), (8, [40], 4100, 129)])
+def test_value_ring_depths(v_stages, hq, ctx, cs, p):
+    """Both value-ring depths give results within tolerance of the oracle and
+    identical to each other (the ring depth changes no arithmetic)."""
+    from paper_2609_38386_gb300 import MX_OPT_V_STAGES
+    case = Case(hq, ctx, chunk_start=cs, p_t=p, seed=v_stages + cs + p)
+    res = case.run_gpu(options={MX_OPT_V_STAGES: v_stages})
+    _ok(case.check(res))
+    other = case.run_gpu(options={MX_OPT_V_STAGES: 5 - v_stages})
+    np.testing.assert_array_equal(res["out"], other["out"])
+
+
+def test_value_ring_option_rejects_other_depths():
+    import paper_2609_38386_gb300 as pkg
+    from paper_2609_38386_gb300 import MX_OPT_V_STAGES
+    ctx = pkg.Context(num_q_heads=16, num_kv_heads=8, num_pages=64, num_seqs=4, max_pages_per_seq=16,
+                      max_tokens=256, max_decodes=4)
+    for bad in (1, 4, -1):
+        with pytest.raises(pkg.MxError):
+            ctx.set_option(MX_OPT_V_STAGES, bad)
+    ctx.set_option(MX_OPT_V_STAGES, 0)
+    ctx.close()
+
+
 def test_prefill_auto_pieces_long_context():
     # a short chunk deep into a long prompt: the planner splits its tiles
     case = Case(16, [2000, 40], chunk_start=6000, p_t=200, seed=8)
