@@ -932,20 +932,35 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
                 if (cc >= nvalid)
                     sv[cc] = 0xFF800000u;
         }
-        const float mx = row_max(sv);
-        const float m_new = fmaxf(m_run, mx * sl);   // log2 domain
-        const bool rescale = m_new > m_run + 8.0f;
-        const float m_use = rescale ? m_new : m_run;
-        // P over the first 64 columns of S (the A operand of P.V)
-        const float rs = few_keys ? row_exp_store<true>(sv, sl, -m_use, tS) : row_exp_store<false>(sv, sl, -m_use, tS);
-        // FA4-style lazy rescale: O moves only when the row max grows by more
-        // than 8 in log2 units.  O_e is stable here: sfull of this tile was
-        // committed after O_e += P_e V of the previous tile, and the next P.V
-        // waits for this tile's P.  tcgen05.ld/st are warp-collective, so the
-        // whole warp rescales when any of its rows must (alpha = 1 for the
-        // others): a branch taken by some lanes only would run them in a
-        // diverged warp.
-        if (i > 0 && __any_sync(0xffffffffu, rescale)) {
+        // FA4-style lazy rescale: the running max m (log2 domain) moves only
+        // when a row's max exceeds it by more than 8, so every weight of P is
+        // at most 2^8.  From the second tile on P is first computed with m as
+        // it stands, without the row max: a tile sum of at most 2^8 shows
+        // that no weight exceeds 2^8, which is all the lazy rule would have
+        // checked (m stays), so the result is the same.  Otherwise the warp
+        // takes the full path: row max, new m where it grew by more than 8, P
+        // computed again (the same bits in the rows whose m stays).  P goes
+        // over the first 64 columns of S (the A operand of P.V).
+        auto exp_store = [&](float m) {
+            return few_keys ? row_exp_store<true>(sv, sl, -m, tS) : row_exp_store<false>(sv, sl, -m, tS);
+        };
+        float m_use = m_run, rs = 0.f;
+        bool rescale = false, resc = false;
+        if (i > 0)
+            rs = exp_store(m_run);
+        if (i == 0 || __any_sync(0xffffffffu, !(rs <= 256.0f))) {
+            const float m_new = fmaxf(m_run, row_max(sv) * sl);
+            rescale = m_new > m_run + 8.0f;
+            m_use = rescale ? m_new : m_run;
+            rs = exp_store(m_use);
+            resc = i > 0 && __any_sync(0xffffffffu, rescale);
+        }
+        // O_e is stable here: sfull of this tile was committed after O_e +=
+        // P_e V of the previous tile, and the next P.V waits for this tile's
+        // P.  tcgen05.ld/st are warp-collective, so the whole warp rescales
+        // when any of its rows must (alpha = 1 for the others): a branch
+        // taken by some lanes only would run them in a diverged warp.
+        if (resc) {
             const float alpha = rescale ? ex2(m_run - m_use) : 1.0f;
 #pragma unroll
             for (int gq = 0; gq < 4; ++gq) {
