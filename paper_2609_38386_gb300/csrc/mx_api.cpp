@@ -327,19 +327,8 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
 
     int split = k.split_keys_opt;
     if (split <= 0) {
-        // Each split pays a fixed start-up and merge cost, so splits are as long
-        // as load balance allows: about 1.5 per SM for a decode-only iteration.
-        // Beside prefill tiles, which hold SMs from the start, the decode
-        // splits must fill around them: the fewer the query tiles, the finer
-        // (3.5 per SM beside one tile, 3 beside 2, 2 beside 3, 1 from 4 on; a
-        // sweep of 1024-4096-key splits over the 0.6B sweep's chunk sizes put
-        // the optimum there).  With independent layers (MX_OPT_PDL = 2) the
-        // next layer fills the tail, so the splits stay long.
-        double per_sm = 1.5;
-        if (n_qt > 0) {
-            static const double kBeside[3] = {3.5, 3.0, 2.0};
-            per_sm = k.pdl == 2 ? 1.0 : (n_qt <= 3 ? kBeside[n_qt - 1] : 1.0);
-        }
+        // splits per SM: the rule of decode_splits_per_sm (mx_internal.h)
+        const double per_sm = decode_splits_per_sm(n_qt, k.pdl == 2, total_keys, k.num_sms);
         const int64_t target_items = std::max<int64_t>(1, (int64_t)(per_sm * k.num_sms));
         int64_t s = (total_keys + target_items - 1) / target_items;
         s = (s + 127) / 128 * 128;

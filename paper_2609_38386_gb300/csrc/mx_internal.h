@@ -57,6 +57,30 @@ __host__ __device__ constexpr int smem_total_bytes(int v_stages)
 constexpr int kSmemTotalMax = smem_total_bytes(kVStagesMax);
 static_assert(kSmemTotalMax <= 227 * 1024, "shared memory per CTA");
 
+// Decode splits per SM that the split length aims at (total keys / (this x
+// SMs)).  Each split pays a fixed start-up and merge cost, so splits are as
+// long as load balance allows: about 1.5 per SM for a decode-only launch.
+// Beside prefill items, which hold SMs from the start, the decode splits
+// must fill around them: the fewer the query tiles, the finer (3.5 per SM
+// beside one tile, 3 beside 2, 2 beside 3, 1 from 4 on), and at least 3
+// when an SM's share of the decode keys is under 8192 (a longer split would
+// be most of that share, and the last ones the launch's tail: on the
+// Qwen3-0.6B sweep, 1024-key splits beat one per SM by up to 9 %, while the
+// 8B and 32B sweeps, with 10K and 37K keys per SM, were best unchanged).
+// With independent layers the next layer fills the tail: 1 per SM.
+inline double decode_splits_per_sm(int n_qt, bool independent_layers, long long total_keys, int num_sms)
+{
+    if (n_qt <= 0)
+        return 1.5;
+    if (independent_layers)
+        return 1.0;
+    const double beside[3] = {3.5, 3.0, 2.0};
+    double k = n_qt <= 3 ? beside[n_qt - 1] : 1.0;
+    if (total_keys < 8192LL * num_sms && k < 3.0)
+        k = 3.0;
+    return k;
+}
+
 // Launch rule for the V ring depth: three stages when the launch's prefill
 // tensor work (flops) is at least 150 times its decode key/value bytes (at
 // the measured peaks, about 0.65 of the decode streaming time).

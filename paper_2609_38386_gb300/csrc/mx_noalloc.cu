@@ -215,8 +215,7 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     total_keys *= hkv;
     int split;
     {
-        static const double kBeside[3] = {3.5, 3.0, 2.0};
-        const double per_sm = n_qt == 0 ? 1.5 : (n_qt <= 3 ? kBeside[n_qt - 1] : 1.0);
+        const double per_sm = decode_splits_per_sm(n_qt, false, total_keys, st->num_sms);
         const int64_t target = std::max<int64_t>(1, (int64_t)(per_sm * st->num_sms));
         int64_t sk = (total_keys + target - 1) / target;
         sk = (sk + 127) / 128 * 128;
