@@ -178,6 +178,26 @@ int mx_iteration(mx_ctx *ctx, const mx_iter_desc *desc, int32_t n_layers,
                  const mx_layer_bufs *layers, float *device_us_out,
                  void *stream);
 
+/* mx_iteration replayed from a CUDA graph (the paper runs its iterations
+ * under CUDA graphs, §4.1): the plan upload and the n_layers launches are
+ * captured once into a graph, and each call only writes the new plan into
+ * the context's replay slot and launches the graph, so the host cost per
+ * call does not grow with n_layers.  The launches read the plan's counts
+ * from device memory, and their TMA descriptors span the buffers'
+ * capacity: each layer's q, k, v and out must hold max_tokens rows of the
+ * context (rows past the call's tokens are read but do not affect the
+ * results).  The graph is captured again when any of layers[0..n_layers),
+ * desc's page_table or slots pointer, MX_OPT_GRID, MX_OPT_PDL,
+ * MX_OPT_WAIT_LIMIT_US or MX_OPT_TEST_STALL_BLOCK differs from the last
+ * capture (one graph is kept per value-ring depth, see MX_OPT_V_STAGES); the
+ * capture happens inside this call, on a stream of the context, and is
+ * not itself capturable.  A call waits until the previous replay has read
+ * its plan.  Results are identical to mx_iteration's; device_us_out, the
+ * error word and the return codes as for mx_iteration. */
+int mx_iteration_graph(mx_ctx *ctx, const mx_iter_desc *desc, int32_t n_layers,
+                       const mx_layer_bufs *layers, float *device_us_out,
+                       void *stream);
+
 /* Wait for `stream`, then read and clear the device error word. */
 int mx_sync_status(mx_ctx *ctx, void *stream);
 

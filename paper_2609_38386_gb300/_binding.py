@@ -28,7 +28,7 @@ MX_OPT_V_STAGES = 7
 
 # Names every C-ABI build must export (the declarations of include/mixattn.h).
 EXPORTS = ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",
-           "mx_iteration", "mx_sync_status", "mx_error_detail", "mx_set_option",
+           "mx_iteration", "mx_iteration_graph", "mx_sync_status", "mx_error_detail", "mx_set_option",
            "mx_last_plan", "mx_plan_work", "mx_mixed_attention_noalloc")
 
 
@@ -88,6 +88,8 @@ def load():
                                    ctypes.POINTER(mx_layer_bufs), P],
             "mx_iteration": [P, ctypes.POINTER(mx_iter_desc), i32,
                              ctypes.POINTER(mx_layer_bufs), ctypes.POINTER(ctypes.c_float), P],
+            "mx_iteration_graph": [P, ctypes.POINTER(mx_iter_desc), i32,
+                                   ctypes.POINTER(mx_layer_bufs), ctypes.POINTER(ctypes.c_float), P],
             "mx_sync_status": [P, P],
             "mx_error_detail": [P, ctypes.c_char_p, i32],
             "mx_set_option": [P, i32, i64],
@@ -240,6 +242,16 @@ class Context:
         self._check(self._lib.mx_iteration(self._h, ctypes.byref(desc), n, arr,
                                            ctypes.byref(us) if wait else None,
                                            _stream_handle(stream)))
+        return float(us.value) if wait else None
+
+    def iteration_graph(self, desc, layers, stream=None, wait=True):
+        """As iteration(), replayed from the context's captured graph (each
+        layer's q/k/v/out must hold max_tokens rows)."""
+        arr, n = layers if isinstance(layers, tuple) else self.layer_array(layers)
+        us = ctypes.c_float()
+        self._check(self._lib.mx_iteration_graph(self._h, ctypes.byref(desc), n, arr,
+                                                 ctypes.byref(us) if wait else None,
+                                                 _stream_handle(stream)))
         return float(us.value) if wait else None
 
     def sync_status(self, stream=None):

@@ -18,6 +18,7 @@ namespace mx {
 cudaError_t init_layer_kernel();
 cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stream, bool pdl);
 cudaError_t launch_plan_upload(const void *src, void *dst, size_t bytes, cudaStream_t stream);
+cudaError_t launch_plan_upload_sized(const void *src, void *dst, size_t max_bytes, cudaStream_t stream);
 cudaError_t launch_kv_append(const int32_t *slots, int n_tokens, int hkv, int num_pages,
                              const uint16_t *k, const uint16_t *v, uint16_t *k_pool,
                              uint16_t *v_pool, uint32_t *err, cudaStream_t stream);
@@ -93,6 +94,23 @@ struct mx_ctx {
     // last plan
     int last_items = 0, last_split = 0, last_prefill_items = 0, last_piece_tiles = 0;
     std::string last_error;
+    // Replayed iterations (mx_iteration_graph): a plan slot of fixed layout
+    // (header, decode table, chunk table, items), allocated on first use, and
+    // one captured graph per V ring depth.
+    uint8_t *gplan_dev = nullptr, *gplan_host = nullptr;
+    const void *gplan_host_dev = nullptr;
+    size_t gplan_bytes = 0;
+    cudaEvent_t gdone = nullptr;   // the last replay has finished (its plan was read)
+    bool gdone_used = false;
+    cudaStream_t cap_stream = nullptr;
+    struct Graph {
+        // what the captured launches hold as constants: a change re-captures
+        std::vector<mx_layer_bufs> layers;
+        const int32_t *page_table = nullptr, *slots = nullptr;
+        int grid = 0, pdl = -1, stall_block = -1;
+        uint64_t wait_ns = 0;
+        cudaGraphExec_t exec = nullptr;
+    } graphs[2];   // [v_stages - 2]
 };
 
 namespace {
@@ -542,11 +560,14 @@ int encode_map(mx_ctx *c, CUtensorMap *m, const void *base, int rank, const cuui
 }
 
 int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const Plan &pl,
-                LayerParams *P, int set)
+                LayerParams *P, int set, const PlanHeader *hdr = nullptr)
 {
     const mx_geom &g = c->g;
     std::memset(P, 0, sizeof *P);
-    const int n_tok = (int)token_count(d);
+    // a replayed launch's maps span the buffers' capacity (its token count
+    // changes from one replay to the next)
+    const int n_tok = hdr ? g.max_tokens : (int)token_count(d);
+    P->hdr = hdr;
     P->q = static_cast<const uint16_t *>(b->q);
     P->k = static_cast<const uint16_t *>(b->k);
     P->v = static_cast<const uint16_t *>(b->v);
@@ -576,7 +597,7 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->num_pages = g.num_pages;
     P->max_pages = g.max_pages_per_seq;
     P->split_keys = pl.split_keys;
-    P->has_prefill = pl.n_prefill > 0 ? 1 : 0;
+    P->has_prefill = (pl.n_prefill > 0 || hdr) ? 1 : 0;
     P->v_stages = pl.v_stages;
     P->scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     P->timeout_ns = c->wait_limit_ns;
@@ -805,6 +826,17 @@ int mx_destroy(mx_ctx *c)
         if (c->slot_done[s])
             cudaEventDestroy(c->slot_done[s]);
     }
+    for (mx_ctx::Graph &gr : c->graphs)
+        if (gr.exec)
+            cudaGraphExecDestroy(gr.exec);
+    if (c->gplan_host)
+        cudaFreeHost(c->gplan_host);
+    if (c->gplan_dev)
+        cudaFree(c->gplan_dev);
+    if (c->gdone)
+        cudaEventDestroy(c->gdone);
+    if (c->cap_stream)
+        cudaStreamDestroy(c->cap_stream);
     if (c->up_stream)
         cudaStreamDestroy(c->up_stream);
     if (c->ev_start)
@@ -915,6 +947,164 @@ int mx_iteration(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_la
     }
     if (work && (rc = release_slot(c, pl, st)))
         return rc;
+    if (!timed)
+        return MX_OK;
+    if ((e = cudaEventRecord(c->ev_end, st)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventRecord(end)");
+    if ((e = cudaEventSynchronize(c->ev_end)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventSynchronize(end)");
+    float ms = 0.f;
+    if ((e = cudaEventElapsedTime(&ms, c->ev_start, c->ev_end)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventElapsedTime");
+    *device_us_out = ms * 1000.0f;
+    return read_error_word(c);
+}
+
+namespace {
+
+// Fixed layout of the replay plan slot: header, decode table (max_decodes),
+// chunk table (kMaxPrefills), items (max_items).
+size_t gplan_dec_off() { return sizeof(PlanHeader); }
+size_t gplan_pre_off(const mx_ctx *c) { return gplan_dec_off() + (size_t)std::max(c->g.max_decodes, 1) * sizeof(DecodeInfo); }
+size_t gplan_items_off(const mx_ctx *c) { return gplan_pre_off(c) + (size_t)kMaxPrefills * sizeof(PrefillInfo); }
+
+int graph_setup(mx_ctx *c)
+{
+    if (c->gplan_dev)
+        return MX_OK;
+    const size_t bytes = gplan_items_off(c) + (size_t)c->max_items * sizeof(int4);
+    cudaError_t e;
+    if ((e = cudaMalloc(&c->gplan_dev, bytes)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaMalloc(replay plan)");
+    if ((e = cudaMallocHost(&c->gplan_host, bytes)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaMallocHost(replay plan)");
+    void *dv = nullptr;
+    if ((e = cudaHostGetDevicePointer(&dv, c->gplan_host, 0)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaHostGetDevicePointer(replay plan)");
+    c->gplan_host_dev = dv;
+    if ((e = cudaEventCreateWithFlags(&c->gdone, cudaEventDisableTiming)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventCreate(replay)");
+    if ((e = cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaStreamCreate(capture)");
+    c->gplan_bytes = bytes;
+    return MX_OK;
+}
+
+// Capture the plan upload and the n_layers layer launches of a replayed
+// iteration with V ring depth v_stages into a graph.
+int graph_capture(mx_ctx *c, const mx_iter_desc *d, int n_layers, const mx_layer_bufs *layers, int v_stages,
+                  int grid, cudaGraphExec_t *out)
+{
+    Plan pl;
+    pl.v_stages = v_stages;
+    pl.n_prefill = 1;
+    pl.items_dev = reinterpret_cast<const int4 *>(c->gplan_dev + gplan_items_off(c));
+    pl.dec_dev = reinterpret_cast<const DecodeInfo *>(c->gplan_dev + gplan_dec_off());
+    pl.pre_dev = reinterpret_cast<const PrefillInfo *>(c->gplan_dev + gplan_pre_off(c));
+    const PlanHeader *hdr = reinterpret_cast<const PlanHeader *>(c->gplan_dev);
+    std::vector<LayerParams> params((size_t)n_layers);
+    for (int l = 0; l < n_layers; ++l) {
+        int rc = make_params(c, d, layers + l, pl, &params[l], l % kWorkSets, hdr);
+        if (rc)
+            return rc;
+        params[l].early_start = (c->pdl == 2 && grid == c->num_sms) ? 1 : 0;
+    }
+    cudaError_t e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "cudaStreamBeginCapture");
+    cudaError_t le = launch_plan_upload_sized(c->gplan_host_dev, c->gplan_dev, c->gplan_bytes, c->cap_stream);
+    for (int l = 0; le == cudaSuccess && l < n_layers; ++l)
+        le = launch_mixed_layer(params[l], grid, c->cap_stream, c->pdl != 0 && l > 0);
+    cudaGraph_t graph = nullptr;
+    e = cudaStreamEndCapture(c->cap_stream, &graph);
+    if (le != cudaSuccess || e != cudaSuccess) {
+        if (graph)
+            cudaGraphDestroy(graph);
+        return cuda_fail(c, le != cudaSuccess ? le : e, "capture of the iteration");
+    }
+    e = cudaGraphInstantiate(out, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess)
+        return cuda_fail(c, e, "cudaGraphInstantiate");
+    return MX_OK;
+}
+
+}  // namespace
+
+int mx_iteration_graph(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const mx_layer_bufs *layers,
+                       float *device_us_out, void *stream)
+{
+    int rc = validate(c, d);
+    if (rc)
+        return rc;
+    if (n_layers <= 0 || !layers)
+        return fail(c, MX_EINVAL, "bad n_layers / layers");
+    // the captured launches read the buffers up to their capacity
+    for (int l = 0; l < n_layers; ++l)
+        if ((rc = validate_bufs(c, layers + l, std::max(c->g.max_tokens, 1))))
+            return rc;
+    if (token_count(d) == 0) {
+        if (device_us_out)
+            *device_us_out = 0.f;
+        return MX_OK;
+    }
+    DeviceGuard guard(c->device);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if ((rc = graph_setup(c)))
+        return rc;
+    cudaError_t e;
+    // the host plan may be rewritten once the last replay has read it
+    if (c->gdone_used && (e = cudaEventSynchronize(c->gdone)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventSynchronize(replay)");
+    PlanHeader *h = reinterpret_cast<PlanHeader *>(c->gplan_host);
+    DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(c->gplan_host + gplan_dec_off());
+    PrefillInfo *pre = reinterpret_cast<PrefillInfo *>(c->gplan_host + gplan_pre_off(c));
+    int4 *items = reinterpret_cast<int4 *>(c->gplan_host + gplan_items_off(c));
+    const PlanKnobs knobs{c->num_sms, c->split_keys_opt, c->piece_tiles_opt, c->pdl, c->max_items, c->v_stages_opt};
+    WorkList wl;
+    if ((rc = build_work_list(c->g, d, knobs, dec, pre, items, &wl, &c->last_error)))
+        return rc;
+    std::memset(h, 0, sizeof *h);
+    h->n_items = wl.n_items;
+    h->n_decodes = d->n_decodes;
+    h->n_prefills = wl.n_prefills;
+    h->has_prefill = wl.n_prefill > 0 ? 1 : 0;
+    h->words = (int32_t)((gplan_items_off(c) + (size_t)wl.n_items * sizeof(int4)) / sizeof(int4));
+    c->last_items = wl.n_items;
+    c->last_split = wl.split_keys;
+    c->last_prefill_items = wl.n_prefill;
+    c->last_piece_tiles = wl.piece_tiles;
+
+    // the graph of this layer array, ring depth, grid and launch order
+    const int grid = c->grid_opt > 0 ? c->grid_opt : c->num_sms;
+    mx_ctx::Graph &gr = c->graphs[wl.v_stages == 3 ? 1 : 0];
+    const bool same = gr.exec && gr.grid == grid && gr.pdl == c->pdl && gr.page_table == d->page_table &&
+                      gr.slots == d->slots && gr.stall_block == c->stall_block && gr.wait_ns == c->wait_limit_ns &&
+                      gr.layers.size() == (size_t)n_layers &&
+                      std::memcmp(gr.layers.data(), layers, sizeof(mx_layer_bufs) * (size_t)n_layers) == 0;
+    if (!same) {
+        if (gr.exec) {
+            cudaGraphExecDestroy(gr.exec);
+            gr.exec = nullptr;
+        }
+        if ((rc = graph_capture(c, d, n_layers, layers, wl.v_stages, grid, &gr.exec)))
+            return rc;
+        gr.layers.assign(layers, layers + n_layers);
+        gr.page_table = d->page_table;
+        gr.slots = d->slots;
+        gr.grid = grid;
+        gr.pdl = c->pdl;
+        gr.stall_block = c->stall_block;
+        gr.wait_ns = c->wait_limit_ns;
+    }
+    const bool timed = device_us_out != nullptr;
+    if (timed && (e = cudaEventRecord(c->ev_start, st)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventRecord(start)");
+    if ((e = cudaGraphLaunch(gr.exec, st)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaGraphLaunch");
+    if ((e = cudaEventRecord(c->gdone, st)) != cudaSuccess)
+        return cuda_fail(c, e, "cudaEventRecord(replay)");
+    c->gdone_used = true;
     if (!timed)
         return MX_OK;
     if ((e = cudaEventRecord(c->ev_end, st)) != cudaSuccess)

@@ -181,6 +181,15 @@ struct DecodeInfo {
     int32_t part_base;  // first partial slot of (this decode, head 0)
 };
 
+// Header of a plan uploaded for a replayed (captured) iteration: the
+// per-iteration counts that the layer kernel then reads from device memory
+// instead of its parameters, and the size of the plan that the upload copies.
+struct PlanHeader {
+    int32_t n_items, n_decodes, n_prefills, has_prefill;
+    int32_t words;         // 16-byte words of the whole plan, this header included
+    int32_t pad[3];
+};
+
 struct LayerParams {
     CUtensorMap tm_q;      // 3-D {128, Hq, n_tokens}, box {64, 1, 128}
     CUtensorMap tm_k;      // 3-D {128, Hkv, n_tokens}, box {64, 1, 128}
@@ -218,6 +227,10 @@ struct LayerParams {
     float scale_log2;      // log2(e) / sqrt(head_dim)
     uint64_t timeout_ns;   // bound on every in-kernel wait
     int32_t stall_block;   // fault injection: this block's first wait never completes (-1 = none)
+    // Replayed launches: the plan header (counts above are then ignored),
+    // and the tensor maps span the buffers' capacity rather than the
+    // iteration's tokens.  Null for ordinary launches.
+    const PlanHeader *hdr;
 };
 
 }  // namespace mx

@@ -56,6 +56,7 @@ struct Misc {
     int32_t item_idx[2];
     int32_t abort;
     int32_t last;
+    int32_t n_items;                  // work items of the launch
     PrefillInfo pre[kMaxPrefills];    // the launch's prefill chunks
 };
 static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
@@ -498,6 +499,21 @@ __device__ __forceinline__ void clear_uncached_rows(uint32_t dv, int r0)
     fence_proxy_async_smem();
 }
 
+// Zero value rows [r0, r1) of a staged V tile (two SW128 halves).
+__device__ __forceinline__ void zero_v_rows(uint32_t dv, int r0, int r1)
+{
+#pragma unroll 1
+    for (int r = r0; r < r1; ++r)
+#pragma unroll 1
+        for (int hf = 0; hf < 2; ++hf)
+#pragma unroll 1
+            for (int cc = 0; cc < 8; ++cc)
+                asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(dv + hf * kHalfTile + r * 128 + cc * 16),
+                             "r"(0u)
+                             : "memory");
+    fence_proxy_async_smem();
+}
+
 // Row max of the raw scores of one S row held in registers (the scale is
 // positive), 8 independent three-input chains.
 __device__ __forceinline__ float row_max(const uint32_t (&sv)[128])
@@ -776,6 +792,11 @@ __device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs 
             const uint32_t dv = sV + vs_cur * kTileBytes;
             if (a.kt0 + j - 1 == nA - 1 && (cs % kTileN) != 0)
                 clear_uncached_rows(dv, cs - (a.kt0 + j - 1) * kTileN);
+            // A replayed launch's k/v maps span the buffers' capacity, so the
+            // chunk's last own tile may hold stale rows past the iteration's
+            // tokens: their weights are 0, but 0 x NaN is not.
+            if (P.hdr && a.kt0 + j - 1 >= nA && pf.p_t - kTileN * (a.kt0 + j - 1 - nA) < kTileN)
+                zero_v_rows(dv, max(0, pf.p_t - kTileN * (a.kt0 + j - 1 - nA)), kTileN);
             vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
             asm volatile("" : "+l"(vdesc));
         }
@@ -1130,7 +1151,7 @@ __device__ void producer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
     for (;;) {
         item_boundary();
         const int idx = misc->item_idx[buf];
-        if (idx >= P.n_items || misc->abort)
+        if (idx >= misc->n_items || misc->abort)
             break;
         if (tid == 0)
             misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
@@ -1179,7 +1200,7 @@ __device__ void consumer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
     for (;;) {
         item_boundary();
         const int idx = misc->item_idx[buf];
-        if (idx >= P.n_items || misc->abort)
+        if (idx >= misc->n_items || misc->abort)
             break;
         const int4 it = P.items[idx];
         if ((it.x & 0xF) == ITEM_PREFILL) {
@@ -1222,7 +1243,13 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     Misc *misc = reinterpret_cast<Misc *>(smem + smem_data_bytes(P.v_stages));
     const int tid = threadIdx.x, warp = tid >> 5;
 
+    // The launch's counts: from its parameters, or (a replayed launch) from
+    // the plan header that the upload kernel wrote before the first layer.
+    const PlanHeader *hdr = P.hdr;
+    const int has_prefill = hdr ? hdr->has_prefill : P.has_prefill;
+    const int n_prefills = hdr ? hdr->n_prefills : P.n_prefills;
     if (tid == 0) {
+        misc->n_items = hdr ? hdr->n_items : P.n_items;
         mbar_init(smem_u32(&misc->bar_q), 1);
         for (int b = 0; b < kKStages; ++b) {
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
@@ -1240,7 +1267,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         mbar_init(smem_u32(&misc->bar_never), 1);
         misc->abort = 0;
         fence_mbar_init();
-        if (P.has_prefill) {
+        if (has_prefill) {
             tma_prefetch_desc(&P.tm_q);
             tma_prefetch_desc(&P.tm_k);
             tma_prefetch_desc(&P.tm_v);
@@ -1248,11 +1275,11 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
             tma_prefetch_desc(&P.tm_vpool);
         }
     }
-    if (P.has_prefill && warp == 1) {
+    if (has_prefill && warp == 1) {
         tmem_alloc(smem_u32(&misc->tmem_base), kTmemCols);
         tmem_relinquish();
     }
-    if (tid >= 64 && tid < 64 + P.n_prefills)
+    if (tid >= 64 && tid < 64 + n_prefills)
         misc->pre[tid - 64] = P.pre[tid - 64];
     // Dependent order (early_start = 0): the previous launch in the stream
     // (the previous layer) must have completed, and its writes be visible,
@@ -1284,7 +1311,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = P.has_prefill ? misc->tmem_base : 0u;
+    const uint32_t tmem = has_prefill ? misc->tmem_base : 0u;
 
     if (warp < kProdThreads / 32) {
         regs_dec<kProdRegs>();
@@ -1312,7 +1339,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     tc_fence_before();
     named_sync(kBarItem, kThreads);
     tc_fence_after();
-    if (P.has_prefill && warp == 1)
+    if (has_prefill && warp == 1)
         tmem_dealloc(tmem, kTmemCols);
     if (tid == 0) {
         __threadfence();
@@ -1382,6 +1409,22 @@ __global__ void plan_upload_kernel(const uint4 *__restrict__ src, uint4 *__restr
 {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
         dst[i] = src[i];
+}
+
+// The same for a replayed iteration: the plan's size is read from its
+// header (at most max_words words).
+__global__ void plan_upload_sized_kernel(const uint4 *__restrict__ src, uint4 *__restrict__ dst, int max_words)
+{
+    const int n = min(reinterpret_cast<const PlanHeader *>(src)->words, max_words);
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+        dst[i] = src[i];
+}
+
+cudaError_t launch_plan_upload_sized(const void *src, void *dst, size_t max_bytes, cudaStream_t stream)
+{
+    plan_upload_sized_kernel<<<8, 256, 0, stream>>>(static_cast<const uint4 *>(src), static_cast<uint4 *>(dst),
+                                                    (int)(max_bytes / sizeof(uint4)));
+    return cudaGetLastError();
 }
 
 cudaError_t launch_plan_upload(const void *src, void *dst, size_t bytes, cudaStream_t stream)

@@ -45,6 +45,7 @@ def test_null_and_geometry_checks_without_gpu(lib):
     assert lib.mx_destroy(None) == 0
     assert lib.mx_mixed_attention(None, None, None, None) == -1
     assert lib.mx_iteration(None, None, 0, None, None, None) == -1
+    assert lib.mx_iteration_graph(None, None, 0, None, None, None) == -1
     assert lib.mx_error_detail(None, None, 0) == -1
     assert lib.mx_set_option(None, 1, 0) == -1
     h = ctypes.c_void_p()
