@@ -407,6 +407,53 @@ def independent_layers_measure(w, steps, ws, device):
             "note": "MX_OPT_PDL=2: consecutive layers overlap (valid only for independent layers)"}
 
 
+def graph_measure(w, device, stride=4):
+    """Host enqueue cost of one iteration call with ordinary launches
+    (mx_iteration) and replayed from a CUDA graph (mx_iteration_graph), on
+    every stride-th iteration of the sweep, with the device times of both.
+    The replayed launches read each layer's q/k/v up to the buffers'
+    capacity, so this needs the lean layout (one buffer per layer, sized for
+    the largest iteration), and one slot buffer that each call refreshes (the
+    graph holds its pointer).  The first pass of each mode (the capture) is
+    not counted."""
+    import time
+
+    import torch
+    slots = torch.full((w.max_tok,), -1, dtype=torch.int32, device=device)
+    idx = list(range(0, len(w.its), stride))
+    gdescs = {}
+    for i in idx:
+        it = w.its[i]
+        gdescs[i] = w.ctx.make_desc(decode_seq_ids=it.decode_seq_ids, decode_ctx_lens=it.decode_ctx_lens,
+                                    prefill_seq_id=it.prefill_seq, chunk_start=it.chunk_start, p_t=it.p_t,
+                                    page_table=w.page_table, slots=slots)
+    out = {"iterations": len(idx), "layers": w.L}
+    for mode in ("iteration", "graph"):
+        enq, dev = [], []
+        for rep in range(2):
+            for i in idx:
+                it = w.its[i]
+                if mode == "graph":
+                    slots[:it.n_tokens].copy_(w.slots[i])
+                torch.cuda.synchronize(device)
+                t0 = time.perf_counter()
+                if mode == "graph":
+                    w.ctx.iteration_graph(gdescs[i], w.layer_arrays[i], wait=False)
+                else:
+                    w.ctx.iteration(w.descs[i], w.layer_arrays[i], wait=False)
+                t1 = time.perf_counter()
+                torch.cuda.synchronize(device)
+                us = (w.ctx.iteration_graph(gdescs[i], w.layer_arrays[i]) if mode == "graph"
+                      else w.ctx.iteration(w.descs[i], w.layer_arrays[i]))
+                if rep:
+                    enq.append((t1 - t0) * 1e6)
+                    dev.append(us)
+        out[mode] = {"enqueue_us_mean": float(np.mean(enq)), "device_us_mean": float(np.mean(dev))}
+    out["note"] = ("host time to enqueue one iteration call (planning, plan write, launches), and device time "
+                   "per iteration; graph = mx_iteration_graph")
+    return out
+
+
 def several_chunks_measure(cfg, peaks, device, layers=28, reps=10):
     """Several prompts' chunks in one iteration (four 512-token chunks of
     four prompts at positions 1024/3072/5120/7168, plus the sweep's 32
@@ -878,6 +925,8 @@ def main():
         line["e2e"] = e2e_measure(w, max(1, min(args.steps, 3)), device)
     if not args.profile:
         line["independent_layers"] = independent_layers_measure(w, max(1, min(args.steps, 3)), ws, device)
+        if args.config in LEAN_CONFIGS or args.lean:
+            line["graph"] = graph_measure(w, device)
     if rank == 0 and ws == 1 and not args.no_cpu and not args.profile:
         line["cpu_baseline"] = cpu_baseline(cfg)
     w.close()
