@@ -317,6 +317,42 @@ int mx_mixed_attention_noalloc(const mx_geom *geom, const mx_iter_desc *desc,
                                const mx_layer_bufs *bufs, void *stream,
                                char *err_buf, int32_t err_len);
 
+/* ------------------------------------------------------------------------
+ * The rest of a Qwen3 decoder layer around mx_mixed_attention (the
+ * whole-model setting of the paper's measurements, §4.1; it sets the share
+ * of L_prefill in Eq. 1's L_t).  Context-free: device pointers to row-major
+ * bf16 tensors (16-byte aligned unless stated), asynchronous on `stream`.
+ * Return MX_OK, MX_EINVAL (arguments; nothing launched) or MX_ECUDA. */
+
+/* y[r] = x[r] / sqrt(mean(x[r]^2) + eps) * w for rows x [rows][dim], w
+ * [dim] (dim a multiple of 8); y may be x. */
+int mx_rms_norm(const void *x, const void *w, void *y, int32_t rows,
+                int32_t dim, float eps, void *stream);
+
+/* From the fused projection qkv [n_tokens][num_q_heads + 2 num_kv_heads][128]
+ * (q heads, then k heads, then v heads): q [n_tokens][num_q_heads][128] and
+ * k [n_tokens][num_kv_heads][128] = the rotary embedding at the token's
+ * position (positions [n_tokens], int32) of the head's RMSNorm over its 128
+ * elements (weights q_norm / k_norm [128]); rotate-half pairing, element i
+ * with i + 64 at frequency theta^(-i/64); v [n_tokens][num_kv_heads][128] =
+ * the v heads.  The outputs are the attention inputs (mx_layer_bufs q, k,
+ * v); pointers 8-byte aligned. */
+int mx_qk_norm_rope(const void *qkv, const void *q_norm, const void *k_norm,
+                    const int32_t *positions, void *q, void *k, void *v,
+                    int32_t n_tokens, int32_t num_q_heads,
+                    int32_t num_kv_heads, float theta, float eps,
+                    void *stream);
+
+/* SwiGLU gate: y[r][j] = silu(gu[r][j]) * gu[r][d_ffn + j] for gate_up
+ * [rows][2 d_ffn] (gate, then up), y [rows][d_ffn], d_ffn a multiple of 8. */
+int mx_silu_mul(const void *gate_up, void *y, int32_t rows, int32_t d_ffn,
+                void *stream);
+
+/* c [m][n] = a [m][k] b [k][n] (+ c when accumulate = 1, e.g. a residual
+ * add), bf16 in and out, fp32 accumulation (a cuBLAS GEMM). */
+int mx_gemm(const void *a, const void *b, void *c, int32_t m, int32_t n,
+            int32_t k, int32_t accumulate, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

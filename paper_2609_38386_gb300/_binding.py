@@ -29,7 +29,8 @@ MX_OPT_V_STAGES = 7
 # Names every C-ABI build must export (the declarations of include/mixattn.h).
 EXPORTS = ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",
            "mx_iteration", "mx_iteration_graph", "mx_sync_status", "mx_error_detail", "mx_set_option",
-           "mx_last_plan", "mx_plan_work", "mx_mixed_attention_noalloc")
+           "mx_last_plan", "mx_plan_work", "mx_mixed_attention_noalloc",
+           "mx_rms_norm", "mx_qk_norm_rope", "mx_silu_mul", "mx_gemm")
 
 
 class MxError(RuntimeError):
@@ -98,6 +99,10 @@ def load():
                                            ctypes.POINTER(mx_layer_bufs), P, ctypes.c_char_p, i32],
             "mx_plan_work": [ctypes.POINTER(mx_geom), ctypes.POINTER(mx_iter_desc), i32, i32, i32, i32,
                              P, i32, P, P, ctypes.c_char_p, i32],
+            "mx_rms_norm": [P, P, P, i32, i32, ctypes.c_float, P],
+            "mx_qk_norm_rope": [P, P, P, P, P, P, P, i32, i32, i32, ctypes.c_float, ctypes.c_float, P],
+            "mx_silu_mul": [P, P, i32, i32, P],
+            "mx_gemm": [P, P, P, i32, i32, i32, i32, P],
         }
         for name, args in sig.items():
             f = getattr(lib, name)
@@ -153,6 +158,48 @@ def _stream_handle(stream):
     if isinstance(stream, int):
         return stream
     return stream.cuda_stream
+
+
+# ------------------------------------------------------------- layer ops
+# The rest of a decoder layer (context-free C-ABI entry points): torch
+# tensors in, argument marshalling only.
+def _op(rc, name):
+    if rc != 0:
+        raise MxError(rc, f"{name} failed ({rc})")
+
+
+def rms_norm(x, w, y, eps, stream=None):
+    """y = x / sqrt(mean(x^2) + eps) * w over the last dim (bf16 as int16)."""
+    rows, dim = x.shape[0], x.shape[-1]
+    assert x.is_contiguous() and y.is_contiguous() and w.numel() == dim and y.shape == x.shape
+    _op(load().mx_rms_norm(x.data_ptr(), w.data_ptr(), y.data_ptr(), rows, dim, float(eps),
+                           _stream_handle(stream)), "mx_rms_norm")
+
+
+def qk_norm_rope(qkv, q_norm, k_norm, positions, q, k, v, num_q_heads, num_kv_heads, theta, eps, stream=None):
+    """q/k/v of the attention from the fused projection (see the header)."""
+    n = qkv.shape[0]
+    assert qkv.is_contiguous() and qkv.numel() == n * (num_q_heads + 2 * num_kv_heads) * 128
+    assert q.is_contiguous() and k.is_contiguous() and v.is_contiguous() and positions.numel() >= n
+    _op(load().mx_qk_norm_rope(qkv.data_ptr(), q_norm.data_ptr(), k_norm.data_ptr(), positions.data_ptr(),
+                               q.data_ptr(), k.data_ptr(), v.data_ptr(), n, num_q_heads, num_kv_heads,
+                               float(theta), float(eps), _stream_handle(stream)), "mx_qk_norm_rope")
+
+
+def silu_mul(gate_up, y, stream=None):
+    rows, d = y.shape[0], y.shape[-1]
+    assert gate_up.is_contiguous() and y.is_contiguous() and gate_up.shape[-1] == 2 * d
+    _op(load().mx_silu_mul(gate_up.data_ptr(), y.data_ptr(), rows, d, _stream_handle(stream)), "mx_silu_mul")
+
+
+def gemm(a, b, c, accumulate=False, stream=None):
+    """c [m][n] (+)= a [m][k] b [k][n], bf16 (as int16), fp32 accumulation."""
+    m, k = a.shape[0], a.numel() // a.shape[0]
+    n = b.shape[-1]
+    assert a.is_contiguous() and b.is_contiguous() and c.is_contiguous()
+    assert b.numel() == k * n and c.numel() == m * n
+    _op(load().mx_gemm(a.data_ptr(), b.data_ptr(), c.data_ptr(), m, n, k, 1 if accumulate else 0,
+                       _stream_handle(stream)), "mx_gemm")
 
 
 class Context:

@@ -13,7 +13,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(HERE, "libmixattn.so")
-SOURCES = ["mx_api.cpp", "mx_layer.cu", "mx_noalloc.cu"]
+SOURCES = ["mx_api.cpp", "mx_layer.cu", "mx_noalloc.cu", "mx_ops.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "-I", os.path.join(ROOT, "include")]
@@ -42,7 +42,7 @@ def build_library(verbose: bool = False) -> str:
         for _, log in res:
             sys.stderr.write(log)
     tmp = LIB + f".tmp{os.getpid()}"
-    cmd = [_nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", tmp] + [o for o, _ in res]
+    cmd = [_nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", tmp] + [o for o, _ in res] + ["-lcublas"]
     subprocess.check_call(cmd)
     os.replace(tmp, LIB)
     return LIB
