@@ -454,6 +454,68 @@ def graph_measure(w, device, stride=4):
     return out
 
 
+# Hidden and MLP widths of the Qwen3 models whose attention geometry each sweep
+# uses (the models' published configurations).
+MODEL_DIMS = {"qwen3-0.6b-attn-28L-chunk-sweep": (1024, 3072),
+              "qwen3-8b-attn-36L-chunk-sweep": (4096, 12288),
+              "qwen3-32b-attn-64L-chunk-sweep": (5120, 25600)}
+
+
+def layer_measure(cfg, device, reps):
+    """Whole decoder layers around the mixed attention (f3): for one
+    iteration of each chunk size of the sweep (at the middle of the prompt)
+    and the decode-only one, the device time of all n_layers layers (RMSNorm,
+    QKV GEMM, QK norm + RoPE, mixed attention with the KV append, O GEMM +
+    residual, RMSNorm, gate/up GEMM, SwiGLU, down GEMM + residual) against
+    the attention alone on the same data.  One layer's random weights serve
+    every layer (the KV pools are per layer); q/k/v are what the layer
+    computes."""
+    import torch
+
+    from paper_2609_38386_gb300.layer import Qwen3Layer, positions_of
+    d, f = MODEL_DIMS[cfg.name]
+    w = Workload(cfg, device, lean=True)
+    g = w.geom
+    layer = Qwen3Layer(d, f, g.hq, g.hkv, seed=cfg.seed + 77, device=device)
+    picks = {}
+    for i, it in enumerate(w.its):
+        if it.chunk_size not in picks or (it.chunk_size and it.chunk_start <= cfg.prompt_len // 2):
+            picks[it.chunk_size] = i
+    rows = []
+    for p, i in sorted(picks.items()):
+        it = w.its[i]
+        n = it.n_tokens
+        pos = torch.from_numpy(positions_of(it)).to(device)
+        x = torch.empty((n, d), dtype=torch.int16, device=device)
+        attns = []
+        for l in range(w.L):
+            q, k, v = w.inputs[i][l]
+            kp, vp = w.pools[l]
+            attns.append({"q": q, "k": k, "v": v, "k_pool": kp, "v_pool": vp, "out": w.outs[l]})
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        full = []
+        for rep in range(reps + 1):
+            x.copy_(torch.randn((n, d), device=device).to(torch.bfloat16).view(torch.int16))
+            torch.cuda.synchronize(device)
+            ev[0].record()
+            for l in range(w.L):
+                layer.forward(w.ctx, w.descs[i], x, pos, attns[l])
+            ev[1].record()
+            torch.cuda.synchronize(device)
+            w.ctx.sync_status()
+            if rep:
+                full.append(ev[0].elapsed_time(ev[1]) * 1e3)
+        att = [w.ctx.iteration(w.descs[i], w.layer_arrays[i]) for _ in range(reps + 1)][1:]
+        fu, au = float(np.median(full)), float(np.median(att))
+        rows.append({"p": it.p_t, "chunk_start": it.chunk_start, "tokens": n, "full_layers_us": fu,
+                     "attention_us": au, "attention_share": au / fu, "tokens_per_s": n / fu * 1e6})
+    w.close()
+    return {"metric": "whole-layer iteration device us (all layers) and the attention share of L_t",
+            "workload": f"{cfg.name.replace('-attn', '')}-full-layers", "d_model": d, "d_ffn": f,
+            "layers": cfg.n_layers, "q_heads": g.hq, "kv_heads": g.hkv, "dtype": "bf16",
+            "data": "synthetic (seeded random weights and activations)", "per_iteration": rows}
+
+
 def several_chunks_measure(cfg, peaks, device, layers=28, reps=10):
     """Several prompts' chunks in one iteration (four 512-token chunks of
     four prompts at positions 1024/3072/5120/7168, plus the sweep's 32
@@ -829,8 +891,9 @@ def main():
     ap.add_argument("--no-side", action="store_true", help="skip the sweeps reported beside the headline")
     ap.add_argument("--lean", action="store_true",
                     help="one q/k/v buffer per layer reused by all iterations (large sweeps)")
-    ap.add_argument("--workload", default="sweep", choices=["sweep", "trace"],
-                    help="trace: the completion-timed DLFP loop vs a fixed chunk cap")
+    ap.add_argument("--workload", default="sweep", choices=["sweep", "trace", "layer"],
+                    help="trace: the completion-timed DLFP loop vs a fixed chunk cap; layer: whole "
+                         "Qwen3 layers (random weights) around the attention on iterations of --config")
     args = ap.parse_args()
 
     ws, rank, local = dist_setup()
@@ -879,6 +942,12 @@ def main():
             print(json.dumps({"metric": "open-loop trace: per-iteration device us P50/P99 and "
                               "ITL/TTFT, completion-timed DLFP vs fixed chunk caps",
                               "workload": "qwen3-0.6b-attn-28L-poisson-trace", **res}))
+        return
+    if args.workload == "layer":
+        if rank == 0:
+            device = torch.device("cuda", local)
+            torch.cuda.set_device(device)
+            print(json.dumps(layer_measure(cfg, device, max(1, args.steps))))
         return
     if ws > 1:
         import torch.distributed as dist
