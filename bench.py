@@ -379,7 +379,7 @@ def e2e_measure(w, steps, device, budget_bytes=12 << 30):
     return res
 
 
-def independent_layers_measure(w, steps, ws, device):
+def independent_layers_measure(w, steps, ws, device, rep=None):
     """The same steps with MX_OPT_PDL=2: layer l+1's CTAs start on the SMs
     layer l frees.  The layers of this workload are independent problems, so
     this is correct here, but a model whose layer l+1 reads layer l's output
@@ -402,7 +402,7 @@ def independent_layers_measure(w, steps, ws, device):
         ms = max_over_ranks(a.elapsed_time(b), ws, device)
     finally:
         w.ctx.set_option(MX_OPT_PDL, 1)
-    return {"value": whole_job_value(w.tokens_per_step, steps, ws, ms), "unit": UNIT,
+    return {"value": whole_job_value(w.tokens_per_step, steps, ws if rep is None else rep, ms), "unit": UNIT,
             "ms_per_step": ms / steps,
             "note": "MX_OPT_PDL=2: consecutive layers overlap (valid only for independent layers)"}
 
@@ -891,6 +891,10 @@ def main():
     ap.add_argument("--no-side", action="store_true", help="skip the sweeps reported beside the headline")
     ap.add_argument("--lean", action="store_true",
                     help="one q/k/v buffer per layer reused by all iterations (large sweeps)")
+    ap.add_argument("--shard", default="none", choices=["none", "kv"],
+                    help="kv (N > 1): each rank runs 1/N of the KV heads (and their query groups) of the "
+                         "same tokens: tensor parallelism of attention, strong scaling, no collective "
+                         "inside attention; default: N independent replicas (weak scaling)")
     ap.add_argument("--workload", default="sweep", choices=["sweep", "trace", "layer"],
                     help="trace: the completion-timed DLFP loop vs a fixed chunk cap; layer: whole "
                          "Qwen3 layers (random weights) around the attention on iterations of --config")
@@ -899,15 +903,24 @@ def main():
     ws, rank, local = dist_setup()
     from synth import workload as wl
     cfg = wl.CONFIGS[args.config]
+    sharded = args.shard == "kv" and ws > 1
+    if sharded:
+        import dataclasses
+        if cfg.hkv % ws:
+            raise SystemExit(f"--shard kv needs the {cfg.hkv} KV heads to divide among {ws} ranks")
+        cfg = dataclasses.replace(cfg, hq=cfg.hq // ws, hkv=cfg.hkv // ws)
+    # every rank processes its own tokens (replicas) or the same tokens (KV-head shards)
+    rep = 1 if sharded else ws
     lean = args.lean or args.config in LEAN_CONFIGS
-    config = {"workload": cfg.name, "q_heads": cfg.hq, "kv_heads": 8, "head_dim": 128,
+    config = {"workload": cfg.name, "q_heads": cfg.hq * (ws if sharded else 1),
+              "kv_heads": cfg.hkv * (ws if sharded else 1), "head_dim": 128,
               "page_size": 16, "layers": cfg.n_layers, "decodes": cfg.n_decodes,
               "decode_ctx": f"{cfg.ctx_dist}[{cfg.ctx_lo},{cfg.ctx_hi}]",
               "prompt_len": cfg.prompt_len, "chunk_sizes": list(cfg.chunk_sizes),
               "iterations_per_step": len(cfg.iterations()),
               "l2": f"inputs larger than L2: each iteration reads {cfg.n_layers} distinct "
                     "per-layer KV pools of several hundred MB or more",
-              "parallelism": f"replicas{ws}"}
+              "parallelism": f"kv-heads{ws}" if sharded else f"replicas{ws}"}
 
     if args.impl == "reference":
         if rank != 0:
@@ -980,11 +993,12 @@ def main():
                                          ClockSampler(gpu_id))
     per_chunk, roofline = summarize(w, it_us, peaks, args.config if not args.profile else None)
     n_it = len(w.its)
-    value = whole_job_value(w.tokens_per_step, args.steps, ws, total_ms)
+    value = whole_job_value(w.tokens_per_step, args.steps, rep, total_ms)
     plan = w.ctx.last_plan()
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "higher_is_better": True, "scaling": "strong" if sharded else "weak", "vs_baseline": None,
+            "dtype": "bf16",
             "data": "synthetic (seeded N(0,1) bf16, random page permutation)",
             "config": config, "roofline": roofline, "per_chunk": per_chunk,
             # per iteration: one plan-upload kernel and one mixed_layer_kernel per layer
@@ -993,7 +1007,7 @@ def main():
     if not args.no_e2e and not args.profile:
         line["e2e"] = e2e_measure(w, max(1, min(args.steps, 3)), device)
     if not args.profile:
-        line["independent_layers"] = independent_layers_measure(w, max(1, min(args.steps, 3)), ws, device)
+        line["independent_layers"] = independent_layers_measure(w, max(1, min(args.steps, 3)), ws, device, rep)
         if args.config in LEAN_CONFIGS or args.lean:
             line["graph"] = graph_measure(w, device)
     if rank == 0 and ws == 1 and not args.no_cpu and not args.profile:

@@ -137,10 +137,11 @@ class SweepConfig:
     seed: int = 0
     first_chunk_start: int | None = None   # single-iteration configs
     single_chunk: int | None = None
+    hkv: int = HKV                          # KV heads (fewer on a rank of a KV-head-sharded run)
 
     @property
     def geom(self) -> Geometry:
-        return Geometry(self.hq)
+        return Geometry(self.hq, self.hkv)
 
     def decode_ctx0(self) -> np.ndarray:
         rng = np.random.default_rng(self.seed)
