@@ -57,6 +57,7 @@ struct Misc {
     int32_t abort;
     int32_t last;
     int32_t n_items;                  // work items of the launch
+    int32_t has_prefill;              // the launch has prefill items (TMEM allocated)
     PrefillInfo pre[kMaxPrefills];    // the launch's prefill chunks
 };
 static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
@@ -762,6 +763,7 @@ __device__ void prefill_load_ring(const LayerParams &P, Misc *misc, const Prefil
 // TMEM columns that P_h(j-1) occupied; it is issued after P_h(j-1) V_{j-1},
 // and the pipe executes in order.  A commit covers every earlier MMA of the
 // thread, so sfull[h] of tile j also says that O_h += P_h V_{j-1} is done.
+template <bool kReplay>
 __device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs &a, uint32_t tmem,
                             uint32_t sbase)
 {
@@ -776,6 +778,13 @@ __device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs 
     // V stage and phase of the tile whose P.V comes next, advanced without a
     // division (the ring depth is a launch parameter)
     uint32_t vs = a.tile0 % vst, vph = (a.tile0 / vst) & 1;
+    // Steps whose V tile needs rows zeroed (-1: none), computed once: clr_a,
+    // the last cached tile, whose rows past chunk_start are not cached yet;
+    // clr_b (replayed launches only), the chunk's last own tile, whose rows
+    // past the chunk may be stale (the k/v maps span the buffers' capacity):
+    // their weights are 0, but 0 x NaN is not.
+    const int clr_a = (cs % kTileN) != 0 ? nA - a.kt0 : -1;
+    const int clr_b = (kReplay && (pf.p_t % kTileN) != 0) ? nA + (pf.p_t - 1) / kTileN - a.kt0 + 1 : -1;
     bool ok = mbar_wait(smem_u32(&misc->bar_q), a.item_no & 1, abort, tmo);
     tc_fence_after();
     const uint64_t qd0 = smem_desc(sbase + kSmemQ, 16, 1024, kSwz128);
@@ -790,13 +799,10 @@ __device__ void prefill_mma(const LayerParams &P, Misc *misc, const PrefillArgs 
                 break;
             }
             const uint32_t dv = sV + vs_cur * kTileBytes;
-            if (a.kt0 + j - 1 == nA - 1 && (cs % kTileN) != 0)
+            if (j == clr_a)
                 clear_uncached_rows(dv, cs - (a.kt0 + j - 1) * kTileN);
-            // A replayed launch's k/v maps span the buffers' capacity, so the
-            // chunk's last own tile may hold stale rows past the iteration's
-            // tokens: their weights are 0, but 0 x NaN is not.
-            if (P.hdr && a.kt0 + j - 1 >= nA && pf.p_t - kTileN * (a.kt0 + j - 1 - nA) < kTileN)
-                zero_v_rows(dv, max(0, pf.p_t - kTileN * (a.kt0 + j - 1 - nA)), kTileN);
+            if (kReplay && j == clr_b)
+                zero_v_rows(dv, pf.p_t % kTileN, kTileN);
             vdesc = smem_desc(dv, kHalfTile, 1024, kSwz128);
             asm volatile("" : "+l"(vdesc));
         }
@@ -1142,6 +1148,7 @@ __device__ __forceinline__ void item_boundary()
 }
 
 // Warpgroup 0's item loop: claims the next item, loads tiles, issues MMAs.
+template <bool kReplay>
 __device__ void producer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1151,7 +1158,7 @@ __device__ void producer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
     for (;;) {
         item_boundary();
         const int idx = misc->item_idx[buf];
-        if (idx >= misc->n_items || misc->abort)
+        if (idx >= (kReplay ? misc->n_items : P.n_items) || misc->abort)
             break;
         if (tid == 0)
             misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
@@ -1176,7 +1183,7 @@ __device__ void producer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
             } else if (warp == 2) {
                 prefill_load_ring(P, misc, a, false, sbase + kSmemV, lane);
             } else if (warp == 1 && lane == 0) {
-                prefill_mma(P, misc, a, tmem, sbase);
+                prefill_mma<kReplay>(P, misc, a, tmem, sbase);
             }
             const uint32_t nT = (uint32_t)(a.kt1 - a.kt0);
             tile_cnt += nT;
@@ -1192,6 +1199,7 @@ __device__ void producer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
 
 // The consumer warpgroups' item loop: softmax and epilogue of prefill items,
 // all of a decode item.
+template <bool kReplay>
 __device__ void consumer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, uint32_t tmem)
 {
     const int tid = threadIdx.x - kProdThreads;     // 0..255
@@ -1200,7 +1208,7 @@ __device__ void consumer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
     for (;;) {
         item_boundary();
         const int idx = misc->item_idx[buf];
-        if (idx >= misc->n_items || misc->abort)
+        if (idx >= (kReplay ? misc->n_items : P.n_items) || misc->abort)
             break;
         const int4 it = P.items[idx];
         if ((it.x & 0xF) == ITEM_PREFILL) {
@@ -1235,6 +1243,9 @@ __device__ void consumer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
 }
 
 // ---------------------------------------------------------------------------
+// kReplay: a launch replayed from a graph (P.hdr holds the plan's counts);
+// compiled apart so that the ordinary launch carries none of its code.
+template <bool kReplay>
 __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_constant__ LayerParams P)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -1245,11 +1256,12 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
 
     // The launch's counts: from its parameters, or (a replayed launch) from
     // the plan header that the upload kernel wrote before the first layer.
-    const PlanHeader *hdr = P.hdr;
+    const PlanHeader *hdr = kReplay ? P.hdr : nullptr;
     const int has_prefill = hdr ? hdr->has_prefill : P.has_prefill;
     const int n_prefills = hdr ? hdr->n_prefills : P.n_prefills;
     if (tid == 0) {
         misc->n_items = hdr ? hdr->n_items : P.n_items;
+        misc->has_prefill = has_prefill;   // read again at the end (not kept in a register)
         mbar_init(smem_u32(&misc->bar_q), 1);
         for (int b = 0; b < kKStages; ++b) {
             mbar_init(smem_u32(&misc->bar_kfull[b]), 1);
@@ -1315,10 +1327,10 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
 
     if (warp < kProdThreads / 32) {
         regs_dec<kProdRegs>();
-        producer_loop(P, smem, misc, tmem);
+        producer_loop<kReplay>(P, smem, misc, tmem);
     } else {
         regs_inc<kConsRegs>();
-        consumer_loop(P, smem, misc, tmem);
+        consumer_loop<kReplay>(P, smem, misc, tmem);
     }
     // Every role left its loop at the same item boundary.
 
@@ -1339,7 +1351,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     tc_fence_before();
     named_sync(kBarItem, kThreads);
     tc_fence_after();
-    if (has_prefill && warp == 1)
+    if (misc->has_prefill && warp == 1)
         tmem_dealloc(tmem, kTmemCols);
     if (tid == 0) {
         __threadfence();
@@ -1384,7 +1396,11 @@ __global__ void kv_append_kernel(const int32_t *__restrict__ slots, int n_tokens
 // Host-side launchers (called from mx_api.cpp)
 cudaError_t init_layer_kernel()
 {
-    return cudaFuncSetAttribute(mixed_layer_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(mixed_layer_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmemTotalMax);
+    if (e != cudaSuccess)
+        return e;
+    return cudaFuncSetAttribute(mixed_layer_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 kSmemTotalMax);
 }
 
@@ -1400,7 +1416,8 @@ cudaError_t launch_mixed_layer(const LayerParams &P, int grid, cudaStream_t stre
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 1 : 0;
-    return cudaLaunchKernelEx(&cfg, mixed_layer_kernel, P);
+    return P.hdr ? cudaLaunchKernelEx(&cfg, mixed_layer_kernel<true>, P)
+                 : cudaLaunchKernelEx(&cfg, mixed_layer_kernel<false>, P);
 }
 
 // Plan upload: the work list and decode table, read by the GPU from mapped
