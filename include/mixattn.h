@@ -241,6 +241,15 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
  * per SM instead of 192, and the smaller L1 slows decode-heavy launches.
  * Results are the same either way. */
 #define MX_OPT_V_STAGES 7
+/* MX_OPT_DECODE_CTAS: how many CTAs of a launch with both prefill and decode
+ * items start on the decode items (the others start on the prefill items,
+ * and each CTA turns to the other kind once its own runs out), so that
+ * decode splits stream from HBM on some SMs while prefill tiles occupy the
+ * tensor cores of the rest.  0 = automatic (the decode's share of the
+ * launch's time at the HBM and tensor rates), -1 = none (every CTA takes
+ * prefill items first), k = the first k CTAs (at most 65535).  Results are
+ * the same for every value. */
+#define MX_OPT_DECODE_CTAS 8
 int mx_set_option(mx_ctx *ctx, int32_t option, int64_t value);
 
 /* Number of work items and decode split length chosen for the last planned

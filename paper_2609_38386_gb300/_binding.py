@@ -25,6 +25,7 @@ MX_OPT_PDL = 4
 MX_OPT_WAIT_LIMIT_US = 5
 MX_OPT_TEST_STALL_BLOCK = 6
 MX_OPT_V_STAGES = 7
+MX_OPT_DECODE_CTAS = 8
 
 # Names every C-ABI build must export (the declarations of include/mixattn.h).
 EXPORTS = ("mx_create", "mx_destroy", "mx_kv_append", "mx_mixed_attention",

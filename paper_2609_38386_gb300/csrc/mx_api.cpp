@@ -90,6 +90,7 @@ struct mx_ctx {
     uint64_t wait_limit_ns = kTimeoutNs;  // MX_OPT_WAIT_LIMIT_US
     int stall_block = -1;                 // MX_OPT_TEST_STALL_BLOCK - 1
     int v_stages_opt = 0;                 // MX_OPT_V_STAGES (0 = automatic)
+    int dec_ctas_opt = 0;                 // MX_OPT_DECODE_CTAS (0 = automatic, -1 = none)
     size_t merge_bytes = 0, pre_cnt_bytes = 0;
     // last plan
     int last_items = 0, last_split = 0, last_prefill_items = 0, last_piece_tiles = 0;
@@ -157,6 +158,7 @@ struct Plan {
     int n_prefill = 0;
     int split_keys = 0;
     int v_stages = 2;
+    int dec_ctas = 0;
     int slot = 0;
     const int4 *items_dev = nullptr;
     const DecodeInfo *dec_dev = nullptr;
@@ -320,9 +322,11 @@ struct PlanKnobs {
     int pdl;               // launch order (MX_OPT_PDL)
     int max_items;         // capacity of the items array
     int v_stages_opt = 0;  // MX_OPT_V_STAGES (0 = automatic)
+    int dec_ctas_opt = 0;  // MX_OPT_DECODE_CTAS (0 = automatic, -1 = none)
+    int grid = 0;          // CTAs of the launch (0 = num_sms)
 };
 struct WorkList {
-    int n_items = 0, n_prefill = 0, n_prefills = 0, split_keys = 0, piece_tiles = 0, v_stages = 2;
+    int n_items = 0, n_prefill = 0, n_prefills = 0, split_keys = 0, piece_tiles = 0, v_stages = 2, dec_ctas = 0;
 };
 
 // a1: the per-iteration work list, on the host, into dec[n_decodes] and
@@ -432,8 +436,12 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
                      [](const PItem &a, const PItem &b) { return a.tiles > b.tiles; });
     if ((int64_t)pitems.size() > k.max_items)
         return fail_to(err, MX_ECAPACITY, "%zu prefill items exceed capacity %d", pitems.size(), k.max_items);
-    for (const PItem &x : pitems)
+    std::vector<int> pre_tiles;
+    pre_tiles.reserve(pitems.size());
+    for (const PItem &x : pitems) {
         items[n++] = x.code;
+        pre_tiles.push_back(x.tiles);
+    }
     const int n_prefill = n;
 
     // A decode with more keys than the split size is cut into equal
@@ -484,6 +492,16 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
     out->split_keys = split;
     out->piece_tiles = piece;
     out->v_stages = k.v_stages_opt > 0 ? k.v_stages_opt : choose_v_stages(pre_flops, dec_bytes);
+    // CTAs that start on the decode queue (none without both kinds of item)
+    if (n_prefill == 0 || n == n_prefill || k.dec_ctas_opt < 0)
+        out->dec_ctas = 0;
+    else if (k.dec_ctas_opt > 0)
+        out->dec_ctas = k.dec_ctas_opt;
+    else {
+        std::vector<long long> heap(kMaxGrid);
+        out->dec_ctas = decode_first_ctas(pre_tiles.data(), n_prefill, pre_flops, dec_bytes,
+                                          k.grid > 0 ? k.grid : k.num_sms, heap.data());
+    }
     return MX_OK;
 }
 
@@ -504,7 +522,8 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     PrefillInfo *pre = reinterpret_cast<PrefillInfo *>(host + pre_off);
     const size_t items_off = pre_off + (size_t)kMaxPrefills * sizeof(PrefillInfo);
     int4 *items = reinterpret_cast<int4 *>(host + items_off);
-    const PlanKnobs knobs{c->num_sms, c->split_keys_opt, c->piece_tiles_opt, c->pdl, c->max_items, c->v_stages_opt};
+    const PlanKnobs knobs{c->num_sms,   c->split_keys_opt, c->piece_tiles_opt, c->pdl,
+                          c->max_items, c->v_stages_opt,   c->dec_ctas_opt,    c->grid_opt};
     WorkList wl;
     int rc = build_work_list(c->g, d, knobs, dec, pre, items, &wl, &c->last_error);
     if (rc)
@@ -534,6 +553,7 @@ int plan(mx_ctx *c, const mx_iter_desc *d, cudaStream_t stream, Plan *out)
     out->n_prefill = wl.n_prefill;
     out->split_keys = wl.split_keys;
     out->v_stages = wl.v_stages;
+    out->dec_ctas = wl.dec_ctas;
     out->slot = slot;
     out->items_dev = reinterpret_cast<const int4 *>(c->plan_dev[slot] + items_off);
     out->dec_dev = reinterpret_cast<const DecodeInfo *>(c->plan_dev[slot]);
@@ -588,6 +608,8 @@ int make_params(mx_ctx *c, const mx_iter_desc *d, const mx_layer_bufs *b, const 
     P->work_cnt = w.work_cnt;
     P->err = c->err;
     P->n_items = pl.n_items;
+    P->n_pre_items = pl.n_prefill;
+    P->dec_ctas = pl.dec_ctas;
     P->n_decodes = d->n_decodes;
     P->pre = pl.pre_dev;
     P->n_prefills = pl.n_prefills;
@@ -1060,7 +1082,8 @@ int mx_iteration_graph(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const
     DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(c->gplan_host + gplan_dec_off());
     PrefillInfo *pre = reinterpret_cast<PrefillInfo *>(c->gplan_host + gplan_pre_off(c));
     int4 *items = reinterpret_cast<int4 *>(c->gplan_host + gplan_items_off(c));
-    const PlanKnobs knobs{c->num_sms, c->split_keys_opt, c->piece_tiles_opt, c->pdl, c->max_items, c->v_stages_opt};
+    const PlanKnobs knobs{c->num_sms,   c->split_keys_opt, c->piece_tiles_opt, c->pdl,
+                          c->max_items, c->v_stages_opt,   c->dec_ctas_opt,    c->grid_opt};
     WorkList wl;
     if ((rc = build_work_list(c->g, d, knobs, dec, pre, items, &wl, &c->last_error)))
         return rc;
@@ -1069,6 +1092,8 @@ int mx_iteration_graph(mx_ctx *c, const mx_iter_desc *d, int32_t n_layers, const
     h->n_decodes = d->n_decodes;
     h->n_prefills = wl.n_prefills;
     h->has_prefill = wl.n_prefill > 0 ? 1 : 0;
+    h->n_pre_items = wl.n_prefill;
+    h->dec_ctas = wl.dec_ctas;
     h->words = (int32_t)((gplan_items_off(c) + (size_t)wl.n_items * sizeof(int4)) / sizeof(int4));
     c->last_items = wl.n_items;
     c->last_split = wl.split_keys;
@@ -1179,6 +1204,11 @@ int mx_set_option(mx_ctx *c, int32_t option, int64_t value)
         if (value != 0 && value != 2 && value != 3)
             return fail(c, MX_EINVAL, "MX_OPT_V_STAGES is 0, 2 or 3");
         c->v_stages_opt = (int)value;
+        return MX_OK;
+    case MX_OPT_DECODE_CTAS:
+        if (value < -1 || value > 65535)
+            return fail(c, MX_EINVAL, "MX_OPT_DECODE_CTAS is -1, 0 or a CTA count up to 65535");
+        c->dec_ctas_opt = (int)value;
         return MX_OK;
     default:
         return fail(c, MX_EINVAL, "unknown option %d", option);

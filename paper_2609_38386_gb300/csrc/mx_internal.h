@@ -89,6 +89,70 @@ __host__ __device__ inline int choose_v_stages(double prefill_flops, double deco
     return prefill_flops > 0.0 && prefill_flops >= 150.0 * decode_bytes ? 3 : 2;
 }
 
+// Makespan, in key tiles, of the prefill items (tiles[0..n), in claim
+// order, heaviest first) claimed by m SMs, each taking the next item when it
+// is free (list scheduling; every item also pays kItemStartTiles of
+// start-up).  heap: caller storage for m entries (no allocation).
+constexpr int kItemStartTiles = 2;
+inline long long prefill_makespan(const int *tiles, int n, int m, long long *heap)
+{
+    for (int i = 0; i < m; ++i)
+        heap[i] = 0;   // a min-heap of the SMs' free times (all zero: valid)
+    long long span = 0;
+    for (int i = 0; i < n; ++i) {
+        const long long t = heap[0] + tiles[i] + kItemStartTiles;
+        span = t > span ? t : span;
+        int j = 0;   // replace the root and sift down
+        for (;;) {
+            const int l = 2 * j + 1, r = l + 1;
+            int c = j;
+            long long v = t;
+            if (l < m && heap[l] < v) { c = l; v = heap[l]; }
+            if (r < m && heap[r] < v) { c = r; v = heap[r]; }
+            if (c == j)
+                break;
+            heap[j] = heap[c];
+            j = c;
+        }
+        heap[j] = t;
+    }
+    return span;
+}
+
+// Launch rule for the CTAs that start on the decode queue (the others start
+// on the prefill queue).  Prefill items are long and few per SM, so SMs
+// taken from them must not lengthen their schedule: D is the largest count
+// up to kMaxDecodeFirst for which the prefill makespan on grid - D SMs stays
+// within 3 % of that on grid SMs.  Only launches with more prefill items
+// than SMs (a single round of prefill items leaves SMs to the decode from
+// the start anyway) and with decode streaming at least a quarter of the
+// launch's time (HBM and tensor rates measured for this kernel on the
+// GB300: 6.8 TB/s, 1.2 PFLOP/s) take any: measured on Qwen3-32B and -8B
+// attention, decode splits running beside the prefill tiles stream more
+// than one SM's share of HBM, up to 4 % faster launches.  heap: kMaxGrid
+// entries of caller storage.
+constexpr int kMaxDecodeFirst = 24;
+constexpr int kMaxGrid = 1024;
+inline int decode_first_ctas(const int *tiles, int n_pre, double prefill_flops, double decode_bytes, int grid,
+                             long long *heap)
+{
+    if (n_pre <= grid || decode_bytes <= 0.0 || grid > kMaxGrid || grid <= kMaxDecodeFirst)
+        return 0;
+    const double t_dec = decode_bytes / 6.8e12, t_pre = prefill_flops / 1.2e15;
+    if (t_dec < 0.25 * (t_dec + t_pre))
+        return 0;
+    const double limit = 1.03 * (double)prefill_makespan(tiles, n_pre, grid, heap);
+    int lo = 0, hi = kMaxDecodeFirst;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) / 2;
+        if ((double)prefill_makespan(tiles, n_pre, grid - mid, heap) <= limit)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    return lo;
+}
+
 // Decode ring: each of the 8 decode warps owns kDecStages stages of one page
 // (K 4 KiB + V 4 KiB).
 constexpr int kPageBytes = kPage * kHeadDim * 2;       // 4 KiB
@@ -187,7 +251,9 @@ struct DecodeInfo {
 struct PlanHeader {
     int32_t n_items, n_decodes, n_prefills, has_prefill;
     int32_t words;         // 16-byte words of the whole plan, this header included
-    int32_t pad[3];
+    int32_t n_pre_items;   // items [0, n_pre_items) are prefill items
+    int32_t dec_ctas;      // CTAs that start on the decode items
+    int32_t pad;
 };
 
 struct LayerParams {
@@ -211,10 +277,13 @@ struct LayerParams {
     float *pre_o;          // [slot][128 rows][128] normalised prefill-piece outputs
     float *pre_lse;        // [slot][128 rows] log2-sum-exp of each piece
     uint32_t *pre_cnt;     // [q tiles * Hq] piece arrival counters (self-resetting)
-    uint32_t *work_cnt;    // [0] next item, [1] CTAs finished (self-resetting)
+    uint32_t *work_cnt;    // [0] next prefill item, [1] CTAs finished, [2] next decode
+                           // item (self-resetting)
     uint32_t *err;         // error word
 
     int32_t n_items;
+    int32_t n_pre_items;   // items [0, n_pre_items) are prefill items, the rest decode items
+    int32_t dec_ctas;      // CTAs [0, dec_ctas) take decode items first, the others prefill items
     int32_t n_decodes;
     const PrefillInfo *pre; // [n_prefills] prefill chunks
     int32_t n_prefills;

@@ -57,6 +57,9 @@ struct Misc {
     int32_t abort;
     int32_t last;
     int32_t n_items;                  // work items of the launch
+    int32_t n_pre;                    // items [0, n_pre) are prefill items
+    int32_t dec_first;                // this CTA draws decode items first (1) or prefill items (0)
+    int32_t queue;                    // thread 0's queue: 0 its first, 1 the other, 2 none left
     int32_t has_prefill;              // the launch has prefill items (TMEM allocated)
     PrefillInfo pre[kMaxPrefills];    // the launch's prefill chunks
 };
@@ -1139,6 +1142,24 @@ __device__ void prefill_merge(const LayerParams &P, Misc *misc, const PrefillInf
         *cnt = 0u;
 }
 
+// The next work item of this CTA (thread 0 only).  The items form two
+// queues: the prefill items [0, n_pre), heaviest first, and the decode items
+// [n_pre, n), longest first.  CTAs below dec_ctas draw from the decode queue
+// first and the others from the prefill queue, and each turns to the other
+// queue once its own is empty: HBM-bound decode splits then stream on some
+// SMs while tensor-bound prefill tiles run on the rest.  n when both are empty.
+__device__ __forceinline__ int32_t claim_item(const LayerParams &P, Misc *misc)
+{
+    while (misc->queue < 2) {
+        const int32_t dec = misc->dec_first ^ misc->queue;
+        const int32_t i = (dec ? misc->n_pre : 0) + (int32_t)atomicAdd(P.work_cnt + 2 * dec, 1u);
+        if (i < (dec ? misc->n_items : misc->n_pre))
+            return i;
+        misc->queue += 1;
+    }
+    return misc->n_items;
+}
+
 // Between items: every thread of the CTA has finished the previous item.
 __device__ __forceinline__ void item_boundary()
 {
@@ -1161,7 +1182,7 @@ __device__ void producer_loop(const LayerParams &P, uint8_t *smem, Misc *misc, u
         if (idx >= (kReplay ? misc->n_items : P.n_items) || misc->abort)
             break;
         if (tid == 0)
-            misc->item_idx[buf ^ 1] = (int32_t)atomicAdd(P.work_cnt, 1u);
+            misc->item_idx[buf ^ 1] = claim_item(P, misc);
         const int4 it = P.items[idx];
         if ((it.x & 0xF) == ITEM_PREFILL) {
             const PrefillArgs a = prefill_args(it, misc, tile_cnt, item_no, sph);
@@ -1261,6 +1282,9 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     const int n_prefills = hdr ? hdr->n_prefills : P.n_prefills;
     if (tid == 0) {
         misc->n_items = hdr ? hdr->n_items : P.n_items;
+        misc->n_pre = hdr ? hdr->n_pre_items : P.n_pre_items;
+        misc->dec_first = (int32_t)blockIdx.x < (hdr ? hdr->dec_ctas : P.dec_ctas) ? 1 : 0;
+        misc->queue = 0;
         misc->has_prefill = has_prefill;   // read again at the end (not kept in a register)
         mbar_init(smem_u32(&misc->bar_q), 1);
         for (int b = 0; b < kKStages; ++b) {
@@ -1305,7 +1329,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
     // that last used this one's set has completed before this one was
     // launched (see the end of the kernel), so work starts at once.
     if (tid == 0) {
-        misc->item_idx[0] = (int32_t)atomicAdd(P.work_cnt, 1u);
+        misc->item_idx[0] = claim_item(P, misc);
         // Fault injection for the bounded waits: the chosen block waits on a
         // barrier that nothing arrives at, with its first item claimed, so
         // the launch ends with that item undone and its counters left set.
@@ -1359,6 +1383,7 @@ __global__ void __launch_bounds__(kThreads, 1) mixed_layer_kernel(const __grid_c
         if (prev == gridDim.x - 1) {
             P.work_cnt[0] = 0u;
             P.work_cnt[1] = 0u;
+            P.work_cnt[2] = 0u;
             __threadfence();
         }
     }

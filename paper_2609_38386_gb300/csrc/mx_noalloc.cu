@@ -248,12 +248,16 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     DecodeInfo *dec = reinterpret_cast<DecodeInfo *>(plan);
     int4 *items = reinterpret_cast<int4 *>(plan + (size_t)kNaMaxDecodes * sizeof(DecodeInfo));
     int n = 0;
-    for (int t = n_qt - 1; t >= 0; --t)
-        for (int h = 0; h < hq; h += nh)
-            items[n++] = prefill_item_code(0, t, h, nh, 0, 1, 0);
-    const int n_prefill = n;
-    // keys of each decode item, for the longest-first order (stable)
+    // key tiles of each prefill item (for the decode-first rule), then keys
+    // of each decode item (for their longest-first order, stable)
     int32_t item_keys[kNaMaxItems];
+    const int n_ahead = (d->chunk_start + kTileN - 1) / kTileN;
+    for (int t = n_qt - 1; t >= 0; --t)
+        for (int h = 0; h < hq; h += nh) {
+            item_keys[n] = n_ahead + t + 1;
+            items[n++] = prefill_item_code(0, t, h, nh, 0, 1, 0);
+        }
+    const int n_prefill = n;
     int part = 0;
     for (int i = 0; i < nd; ++i) {
         const int keys = d->decode_ctx_lens[i] + 1;
@@ -325,8 +329,12 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
     P.max_pages = g->max_pages_per_seq;
     P.split_keys = split;
     P.has_prefill = n_prefill > 0 ? 1 : 0;
-    P.v_stages = choose_v_stages(4.0 * hq * kHeadDim * ((double)p * pre.chunk_start + 0.5 * (double)p * (p + 1)),
-                                 (double)total_keys * kHeadDim * 2 * 2);
+    const double pre_flops = 4.0 * hq * kHeadDim * ((double)p * pre.chunk_start + 0.5 * (double)p * (p + 1));
+    const double dec_bytes = (double)total_keys * kHeadDim * 2 * 2;
+    P.v_stages = choose_v_stages(pre_flops, dec_bytes);
+    P.n_pre_items = n_prefill;
+    long long heap[kMaxGrid];
+    P.dec_ctas = n > n_prefill ? decode_first_ctas(item_keys, n_prefill, pre_flops, dec_bytes, st->num_sms, heap) : 0;
     P.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)kHeadDim));
     P.timeout_ns = 1000000000ull;
     P.stall_block = -1;

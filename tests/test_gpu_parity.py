@@ -247,6 +247,36 @@ def test_value_ring_option_rejects_other_depths():
     ctx.close()
 
 
+@pytest.mark.parametrize("hq,ctx,cs,p", [(16, [900, 3, 64, 5000, 17], 0, 300), (64, [2000, 17, 12000], 1000, 260),
+                                         (8, [40, 700, 700], 4100, 129)])
+def test_decode_first_ctas(hq, ctx, cs, p):
+    """However many CTAs start on the decode queue (none, one, some, all),
+    the results are those of the oracle and identical to each other: the
+    claim order changes which SM runs an item, not its arithmetic."""
+    from paper_2609_38386_gb300 import MX_OPT_DECODE_CTAS
+    case = Case(hq, ctx, chunk_start=cs, p_t=p, seed=hq + cs + p)
+    base = case.run_gpu(options={MX_OPT_DECODE_CTAS: -1})
+    _ok(case.check(base))
+    for d in (0, 1, 37, 65535):
+        res = case.run_gpu(options={MX_OPT_DECODE_CTAS: d})
+        np.testing.assert_array_equal(res["out"], base["out"])
+        np.testing.assert_array_equal(res["k_pool"], base["k_pool"])
+        np.testing.assert_array_equal(res["v_pool"], base["v_pool"])
+
+
+def test_decode_ctas_option_range():
+    import paper_2609_38386_gb300 as pkg
+    from paper_2609_38386_gb300 import MX_OPT_DECODE_CTAS
+    ctx = pkg.Context(num_q_heads=16, num_kv_heads=8, num_pages=64, num_seqs=4, max_pages_per_seq=16,
+                      max_tokens=256, max_decodes=4)
+    for bad in (-2, 65536):
+        with pytest.raises(pkg.MxError):
+            ctx.set_option(MX_OPT_DECODE_CTAS, bad)
+    for good in (-1, 0, 152):
+        ctx.set_option(MX_OPT_DECODE_CTAS, good)
+    ctx.close()
+
+
 def test_prefill_auto_pieces_long_context():
     # a short chunk deep into a long prompt: the planner splits its tiles
     case = Case(16, [2000, 40], chunk_start=6000, p_t=200, seed=8)
