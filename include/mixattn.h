@@ -261,11 +261,13 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  * (the planning step of mx_mixed_attention / mx_iteration, exposed so that
  * schedulers and tests can inspect it).  The paper schedules per iteration a
  * decode set D_t and a prefill chunk of p_t tokens (§2.1, Eq. 1); one launch
- * splits that work into items that its persistent CTAs claim in order:
- * prefill query tiles (128 rows x two query heads of one KV head, or one
- * head when num_q_heads == num_kv_heads; or a key piece of one), heaviest
- * first, then decode splits (one decode x one KV head x a key range),
- * longest first.
+ * splits that work into items in two queues that its persistent CTAs claim
+ * from: prefill query tiles (128 rows x two query heads of one KV head, or
+ * one head when num_q_heads == num_kv_heads; or a key piece of one),
+ * heaviest first, and decode splits (one decode x one KV head x a key
+ * range), longest first.  The first counts[4] CTAs start on the decode
+ * queue, the others on the prefill queue; each turns to the other queue
+ * when its own is empty (MX_OPT_DECODE_CTAS).
  *
  * geom and desc as for mx_create / mx_mixed_attention (desc's page_table and
  * slots are not read and may be NULL); num_sms: the SM count the launch will
@@ -287,7 +289,10 @@ int mx_last_plan(mx_ctx *ctx, int32_t *n_items, int32_t *split_keys,
  *       decode of at most 64 keys (one split, computed exactly in fp32);
  *   decodes  int32 [n_decodes][4]: page-table row, ctx, number of splits,
  *     first partial slot (of head 0; head h uses base + h * splits);
- *   counts   int32 [4]: n_items, prefill items, split_keys, piece_tiles.
+ *   counts   int32 [5]: n_items, prefill items (items [0, prefill items)
+ *     are the prefill queue, the rest the decode queue), split_keys,
+ *     piece_tiles, CTAs that start on the decode queue (the automatic
+ *     choice of MX_OPT_DECODE_CTAS for a grid of num_sms).
  * Returns MX_OK, MX_EINVAL (arguments, geometry, descriptor) or MX_ECAPACITY
  * (the work does not fit max_items or the context's partial workspace), with
  * a message in err_buf (up to err_len bytes) when err_buf is not NULL. */

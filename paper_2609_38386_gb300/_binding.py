@@ -119,7 +119,8 @@ def plan_work(*, num_q_heads, num_kv_heads=8, num_pages, num_seqs, max_pages_per
               pdl=1, max_items=1 << 16):
     """The work list a launch would run (host only, no device): items
     int32 [n, 4] in claim order, decodes int32 [n_decodes, 4] and the counts
-    (n_items, prefill items, split_keys, piece_tiles)."""
+    (n_items, prefill items, split_keys, piece_tiles, CTAs that start on the
+    decode queue)."""
     lib = load()
     geom = mx_geom(num_q_heads, num_kv_heads, 128, 16, num_pages, num_seqs, max_pages_per_seq,
                    max_tokens, max_decodes)
@@ -131,7 +132,7 @@ def plan_work(*, num_q_heads, num_kv_heads=8, num_pages, num_seqs, max_pages_per
                         n_pf, ctypes.cast(pf_arr, ctypes.c_void_p) if pf_arr is not None else None)
     items = np.zeros((max(max_items, 1), 4), np.int32)
     decs = np.zeros((max(len(lens), 1), 4), np.int32)
-    counts = np.zeros(4, np.int32)
+    counts = np.zeros(5, np.int32)
     err = ctypes.create_string_buffer(512)
     rc = lib.mx_plan_work(ctypes.byref(geom), ctypes.byref(desc), int(num_sms), int(split_keys),
                           int(piece_tiles), int(pdl), items.ctypes.data, int(max_items),
@@ -140,7 +141,7 @@ def plan_work(*, num_q_heads, num_kv_heads=8, num_pages, num_seqs, max_pages_per
         raise MxError(rc, err.value.decode(errors="replace"))
     return {"items": items[:counts[0]].copy(), "decodes": decs[:len(lens)].copy(),
             "n_items": int(counts[0]), "n_prefill_items": int(counts[1]),
-            "split_keys": int(counts[2]), "piece_tiles": int(counts[3])}
+            "split_keys": int(counts[2]), "piece_tiles": int(counts[3]), "decode_first_ctas": int(counts[4])}
 
 
 def _ptr(t):

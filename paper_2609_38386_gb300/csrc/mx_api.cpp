@@ -1245,6 +1245,7 @@ int mx_plan_work(const mx_geom *geom, const mx_iter_desc *desc, int32_t num_sms,
             counts[1] = wl.n_prefill;
             counts[2] = wl.split_keys;
             counts[3] = wl.piece_tiles;
+            counts[4] = wl.dec_ctas;
         }
     }
     if (rc != MX_OK && err_buf && err_len > 0) {

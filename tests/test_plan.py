@@ -231,6 +231,55 @@ def test_automatic_splits_and_pieces():
     assert pl["n_prefill_items"] == 16 * 8
 
 
+def _makespan(tiles, m, start=2):
+    """List schedule of items (key tiles, claim order) on m SMs, each item
+    paying `start` tiles of start-up: the latest finish."""
+    import heapq
+    h = [0] * m
+    for t in tiles:
+        heapq.heapreplace(h, h[0] + t + start)
+    return max(h)
+
+
+def test_decode_first_ctas():
+    """CTAs that start on the decode queue: none when the prefill items fit
+    in one round on the SMs, without decodes, or when the decode is a small
+    share of the launch; otherwise at most 24, chosen so that the prefill
+    items' schedule on the remaining SMs is within 3 % of theirs on all SMs."""
+    rng = np.random.default_rng(5)
+    ctxs = [int(c) for c in np.exp(rng.uniform(np.log(1024), np.log(16384), 128))]
+    # 1024 rows at 16384, 64 query heads: 8 tiles x 32 head pairs = 256 items
+    # of 129..136 key tiles, two rounds on 152 SMs and on 128
+    pl = _plan(64, ctxs, 16384, 1024)
+    assert pl["decode_first_ctas"] == 24
+    assert _plan(64, ctxs, 16384, 1024, sms=100)["decode_first_ctas"] <= 24
+    # one round of prefill items (64 on 152 SMs), no decodes, a long chunk
+    # beside a few decodes: none
+    assert _plan(16, ctxs[:32], 4096, 1024)["decode_first_ctas"] == 0
+    assert _plan(64, [], 16384, 1024)["decode_first_ctas"] == 0
+    assert _plan(64, ctxs[:8], 24576, 8192)["decode_first_ctas"] == 0
+    # the defining property over random iterations
+    seen = 0
+    for seed in range(12):
+        r = np.random.default_rng(100 + seed)
+        hq = int(r.choice([16, 32, 64]))
+        nd = int(r.integers(1, 129))
+        cx = [int(c) for c in r.integers(100, 16384, nd)]
+        cs, p = int(r.integers(0, 24576)), int(r.choice([256, 1024, 2048, 4096]))
+        pl = _plan(hq, cx, cs, p)
+        pre, _ = _check(pl, hq, cx, cs, p)
+        n_a = -(-cs // TILE)
+        tiles = [(n_a + d["t"] + 1) * (d["s"] + 1) // d["ns"] - (n_a + d["t"] + 1) * d["s"] // d["ns"]
+                 for d in pre]
+        dq = pl["decode_first_ctas"]
+        assert 0 <= dq <= 24
+        if dq:
+            seen += 1
+            assert len(tiles) > 152
+            assert _makespan(tiles, 152 - dq) <= 1.03 * _makespan(tiles, 152)
+    assert seen > 0
+
+
 def test_partial_workspace_bounds_the_split_count():
     # 128 decodes x 8 heads at 128-key splits would need 128k partial slots:
     # the planner lengthens the splits until they fit
