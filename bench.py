@@ -886,6 +886,9 @@ def main():
     ap.add_argument("--profile", action="store_true",
                     help="small case for ncu: 2 layers, iterations of --profile-chunk only")
     ap.add_argument("--profile-chunk", type=int, default=2048)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run only the first N layers of every iteration (for launch-list captures: "
+                         "each launch does the same work as in the full sweep, on its own layer's pool)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-side", action="store_true", help="skip the sweeps reported beside the headline")
@@ -970,7 +973,7 @@ def main():
     torch.cuda.set_device(device)
     peaks = load_peaks()
 
-    layers = 2 if args.profile else None
+    layers = 2 if args.profile else (args.layers or None)
     w = Workload(cfg, device, seed_offset=replica_seed_offset(rank), layers=layers, lean=lean)
     if lean:
         config["inputs"] = "one q/k/v buffer per layer, reused by every iteration"
@@ -983,6 +986,9 @@ def main():
         w.inputs = [w.inputs[i] for i in keep]
         w.tokens_per_step = sum(it.n_tokens for it in w.its)
         config["workload"] += f"-profile-{w.L}L-p{args.profile_chunk}"
+    elif args.layers:
+        config["workload"] += f"-first-{w.L}L"
+        config["layers"] = w.L
 
     def barrier():
         if ws > 1:
