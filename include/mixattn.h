@@ -101,7 +101,9 @@ typedef struct {
  * ctx; it attends ctx + 1 keys).  prefill_seq_id is the page-table row of the
  * prompt being prefilled (ignored when p_t == 0); its chunk covers positions
  * [chunk_start, chunk_start + p_t) and row j attends keys
- * [0, chunk_start + j].  page_table and slots are DEVICE arrays. */
+ * [0, chunk_start + j].  A sequence takes part at most once per iteration,
+ * as one decode or as one prefill chunk (otherwise MX_EINVAL, nothing
+ * launched).  page_table and slots are DEVICE arrays. */
 typedef struct {
     const int32_t *decode_seq_ids;  /* host  [n_decodes]                  */
     const int32_t *decode_ctx_lens; /* host  [n_decodes]                  */

@@ -252,6 +252,21 @@ int validate_desc(const mx_geom &g, const mx_iter_desc *d, bool need_tables, std
             return fail_to(err, MX_ECAPACITY, "chunk end %lld exceeds %lld page-table slots",
                            (long long)d->chunk_start + d->p_t, (long long)cap);
     }
+    // A sequence takes part once per iteration, as one decode or as one
+    // prefill chunk: two entries of one sequence would append to and read
+    // the same pages in the same launch.
+    {
+        std::vector<int32_t> ids(d->decode_seq_ids, d->decode_seq_ids + d->n_decodes);
+        for (int f = 0; f < d->n_prefills; ++f)
+            ids.push_back(d->prefills[f].seq_id);
+        if (d->n_prefills == 0 && d->p_t > 0)
+            ids.push_back(d->prefill_seq_id);
+        std::sort(ids.begin(), ids.end());
+        const auto rep = std::adjacent_find(ids.begin(), ids.end());
+        if (rep != ids.end())
+            return fail_to(err, MX_EINVAL, "sequence %d appears twice in the iteration (decodes and chunks)",
+                           *rep);
+    }
     if (need_tables && n_tok > 0 && (!d->page_table || !d->slots))
         return fail_to(err, MX_EINVAL, "page_table / slots are null");
     return MX_OK;

@@ -179,6 +179,20 @@ extern "C" int mx_mixed_attention_noalloc(const mx_geom *g, const mx_iter_desc *
         if ((int64_t)d->chunk_start + p > cap)
             return report(err_buf, err_len, MX_ECAPACITY, "chunk exceeds the page table");
     }
+    {
+        // a sequence takes part once: as one decode or as the chunk (two
+        // entries of one sequence would append to and read the same pages)
+        int32_t ids[kNaMaxDecodes + 1];
+        int n_ids = 0;
+        for (int i = 0; i < nd; ++i)
+            ids[n_ids++] = d->decode_seq_ids[i];
+        if (p > 0)
+            ids[n_ids++] = d->prefill_seq_id;
+        std::sort(ids, ids + n_ids);
+        for (int i = 1; i < n_ids; ++i)
+            if (ids[i] == ids[i - 1])
+                return report(err_buf, err_len, MX_EINVAL, "sequence %d appears twice in the iteration", ids[i]);
+    }
     const int n_tok = nd + p;
     if (n_tok == 0)
         return MX_OK;

@@ -66,3 +66,23 @@ def test_null_and_geometry_checks_without_gpu(lib):
         good = mx_geom(16, 8, 128, 16, 10, 1, 4, 8, 1)
         assert lib.mx_create(ctypes.byref(h), ctypes.byref(good), 0) == -6   # MX_EDEVICE
         assert lib.mx_error_detail(None, buf, 256) > 0 and b"device" in buf.value
+
+
+def test_noalloc_rejects_a_repeated_sequence_before_any_cuda_call(lib):
+    """The allocation-free entry point checks its descriptor on the host
+    first: a sequence listed twice (two decodes, or a decode and the chunk)
+    returns MX_EINVAL before any CUDA call, so this runs without a GPU.  The
+    tensor pointers are never dereferenced."""
+    from paper_2609_38386_gb300._binding import mx_geom, mx_iter_desc, mx_layer_bufs
+    import numpy as np
+    geom = mx_geom(16, 8, 128, 16, 100, 4, 8, 0, 0)
+    fake = 1 << 20                                       # aligned, never used
+    bufs = mx_layer_bufs(fake, fake, fake, fake, fake, fake)
+    err = ctypes.create_string_buffer(256)
+    for ids, pseq, p in (([1, 1], -1, 0), ([0, 2], 2, 16)):
+        seqs = np.asarray(ids, np.int32)
+        lens = np.asarray([5, 6], np.int32)
+        desc = mx_iter_desc(seqs.ctypes.data, lens.ctypes.data, 2, pseq, 0, p, fake, fake, 0, None)
+        rc = lib.mx_mixed_attention_noalloc(ctypes.byref(geom), ctypes.byref(desc), ctypes.byref(bufs),
+                                            None, err, 256)
+        assert rc == -1 and b"twice" in err.value, (rc, err.value)

@@ -311,3 +311,21 @@ def test_rejections():
     with pytest.raises(MxError, match="EINVAL"):         # split option not a multiple of 128
         _plan(16, [100], split_keys=100)
 
+
+def test_a_sequence_takes_part_once():
+    """A sequence is one decode or one prefill chunk of an iteration, not
+    two entries: those would append to and read the same pages in one
+    launch.  Each repetition is rejected on the host before any launch."""
+    base = dict(num_q_heads=16, num_pages=1000, num_seqs=4, max_pages_per_seq=64, max_tokens=600,
+                max_decodes=3)
+    with pytest.raises(MxError, match="appears twice"):      # two decodes of sequence 1
+        plan_work(decode_seq_ids=[1, 0, 1], decode_ctx_lens=[5, 6, 7], **base)
+    with pytest.raises(MxError, match="appears twice"):      # a decode and the chunk
+        plan_work(decode_seq_ids=[0, 2], decode_ctx_lens=[5, 6], prefill_seq_id=2, chunk_start=0, p_t=20,
+                  **base)
+    with pytest.raises(MxError, match="appears twice"):      # a decode and one of several chunks
+        plan_work(decode_seq_ids=[0, 3], decode_ctx_lens=[5, 6], prefills=[(1, 0, 10), (3, 0, 10)], **base)
+    # distinct sequences plan; a decode-only descriptor's prefill row is ignored
+    plan_work(decode_seq_ids=[0, 3], decode_ctx_lens=[5, 6], prefills=[(1, 0, 10), (2, 0, 10)], **base)
+    plan_work(decode_seq_ids=[0, 3], decode_ctx_lens=[5, 6], prefill_seq_id=3, p_t=0, **base)
+
