@@ -466,20 +466,55 @@ __device__ void decode_item(const LayerParams &P, uint8_t *smem, Misc *misc, int
     if (!misc->last)
         return;
     __threadfence();
+    // Every partial is read once, eight splits' (lse, 4 columns of O) at a
+    // time with all their loads in flight, the max and the weight sum kept
+    // online (a rescale per group): the merge sits on this split's critical
+    // path, so its loads must not form a chain of round trips.
     const int base = D.part_base + h * nsp;
-    for (int e = tid; e < nrep * kHeadDim; e += kConsThreads) {
-        const int q = e / kHeadDim, d = e % kHeadDim;
-        float M = neg_inf();
-        for (int sp = 0; sp < nsp; ++sp)
-            M = fmaxf(M, __ldcg(P.part_lse + (size_t)(base + sp) * kMaxRep + q));
-        float W = 0.f, O = 0.f;
-        for (int sp = 0; sp < nsp; ++sp) {
-            const float f = ex2(__ldcg(P.part_lse + (size_t)(base + sp) * kMaxRep + q) - M);
-            W += f;
-            O += f * __ldcg(P.part_o + ((size_t)(base + sp) * kMaxRep + q) * kHeadDim + d);
+    for (int e = tid; e < nrep * (kHeadDim / 4); e += kConsThreads) {
+        const int q = e / (kHeadDim / 4), d4 = e % (kHeadDim / 4);
+        float M = neg_inf(), W = 0.f;
+        float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int s0 = 0; s0 < nsp; s0 += 8) {
+            float l[8];
+            float4 o[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int sp = s0 + u;
+                l[u] = neg_inf();
+                o[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (sp < nsp) {
+                    const size_t row = (size_t)(base + sp) * kMaxRep + q;
+                    l[u] = __ldcg(P.part_lse + row);
+                    o[u] = __ldcg(reinterpret_cast<const float4 *>(P.part_o + row * kHeadDim) + d4);
+                }
+            }
+            float mb = M;
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                mb = fmaxf(mb, l[u]);
+            const float c = ex2(M - mb);   // 0 for the first group (M = -inf)
+            W *= c;
+            O.x *= c;
+            O.y *= c;
+            O.z *= c;
+            O.w *= c;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const float f = ex2(l[u] - mb);   // 0 past the last split
+                W += f;
+                O.x += f * o[u].x;
+                O.y += f * o[u].y;
+                O.z += f * o[u].z;
+                O.w += f * o[u].w;
+            }
+            M = mb;
         }
-        __nv_bfloat16 b = __float2bfloat16_rn(O / W);
-        P.out[((size_t)di * P.hq + h * nrep + q) * kHeadDim + d] = *reinterpret_cast<uint16_t *>(&b);
+        const float inv = 1.0f / W;
+        uint2 pk;
+        pk.x = pack_bf16(O.x * inv, O.y * inv);
+        pk.y = pack_bf16(O.z * inv, O.w * inv);
+        reinterpret_cast<uint2 *>(P.out + ((size_t)di * P.hq + h * nrep + q) * kHeadDim)[d4] = pk;
     }
     if (tid == 0)
         P.merge_cnt[di * P.hkv + h] = 0u;
@@ -1098,44 +1133,71 @@ __device__ void prefill_merge(const LayerParams &P, Misc *misc, const PrefillInf
     if (!misc->last)
         return;
     __threadfence();
-    const int r = tid >> 1, half = tid & 1;
-    const int j = kTileM * a.t + r;
-    for (int e = 0; e < a.nh && j < pf.p_t; ++e) {
+    // Consumer warp w merges rows [16 w, 16 w + 16) of the tile, four rows
+    // at a time: a row's 128 columns are one float4 per lane, so every load
+    // reads whole rows (coalesced), and the partials of four pieces of four
+    // rows are in flight together; the max and the weight sum of a row are
+    // kept online over the groups of pieces.
+    const int warp = tid >> 5, lane = tid & 31;
+    for (int e = 0; e < a.nh; ++e) {
         const int base = a.part_base + e * a.ns;
-        float M = neg_inf();
-        for (int s = 0; s < a.ns; ++s)
-            M = fmaxf(M, __ldcg(P.pre_lse + (size_t)(base + s) * kTileM + r));
-        float W = 0.f;
-        for (int s = 0; s < a.ns; ++s)
-            W += ex2(__ldcg(P.pre_lse + (size_t)(base + s) * kTileM + r) - M);
-        const float inv = 1.0f / W;
-        for (int sub = 0; sub < 2; ++sub) {
-            const int d0 = half * 64 + sub * 32;
-            float acc[32];
+        for (int r4 = 0; r4 < kTileM / kWarps; r4 += 4) {
+            const int r0 = warp * (kTileM / kWarps) + r4;
+            float M[4], W[4];
+            float4 acc[4];
 #pragma unroll
-            for (int x = 0; x < 32; ++x)
-                acc[x] = 0.f;
-            for (int s = 0; s < a.ns; ++s) {
-                const float w = ex2(__ldcg(P.pre_lse + (size_t)(base + s) * kTileM + r) - M);
-                const float4 *src =
-                    reinterpret_cast<const float4 *>(P.pre_o + ((size_t)(base + s) * kTileM + r) * kHeadDim + d0);
+            for (int rr = 0; rr < 4; ++rr) {
+                M[rr] = neg_inf();
+                W[rr] = 0.f;
+                acc[rr] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            for (int s0 = 0; s0 < a.ns; s0 += 4) {
+                float l[4][4];
+                float4 v[4][4];
 #pragma unroll
-                for (int x = 0; x < 8; ++x) {
-                    const float4 v = __ldcg(src + x);
-                    acc[4 * x] += w * v.x;
-                    acc[4 * x + 1] += w * v.y;
-                    acc[4 * x + 2] += w * v.z;
-                    acc[4 * x + 3] += w * v.w;
+                for (int rr = 0; rr < 4; ++rr) {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const bool ok = s0 + u < a.ns;
+                        const size_t row = (size_t)(base + s0 + u) * kTileM + r0 + rr;
+                        l[rr][u] = ok ? __ldcg(P.pre_lse + row) : neg_inf();
+                        v[rr][u] = ok ? __ldcg(reinterpret_cast<const float4 *>(P.pre_o + row * kHeadDim) + lane)
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+                    }
+                }
+#pragma unroll
+                for (int rr = 0; rr < 4; ++rr) {
+                    const float mb = fmaxf(fmaxf(M[rr], fmaxf(l[rr][0], l[rr][1])), fmaxf(l[rr][2], l[rr][3]));
+                    const float c = ex2(M[rr] - mb);   // 0 for the first group (M = -inf)
+                    W[rr] *= c;
+                    acc[rr].x *= c;
+                    acc[rr].y *= c;
+                    acc[rr].z *= c;
+                    acc[rr].w *= c;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const float f = ex2(l[rr][u] - mb);   // 0 past the last piece
+                        W[rr] += f;
+                        acc[rr].x += f * v[rr][u].x;
+                        acc[rr].y += f * v[rr][u].y;
+                        acc[rr].z += f * v[rr][u].z;
+                        acc[rr].w += f * v[rr][u].w;
+                    }
+                    M[rr] = mb;
                 }
             }
-            uint4 *dst = reinterpret_cast<uint4 *>(P.out + ((size_t)(pf.token_base + j) * P.hq + a.hq0 + e) *
-                                                              kHeadDim + d0);
 #pragma unroll
-            for (int x = 0; x < 4; ++x)
-                dst[x] = make_uint4(pack_bf16(acc[8 * x] * inv, acc[8 * x + 1] * inv),
-                                    pack_bf16(acc[8 * x + 2] * inv, acc[8 * x + 3] * inv),
-                                    pack_bf16(acc[8 * x + 4] * inv, acc[8 * x + 5] * inv),
-                                    pack_bf16(acc[8 * x + 6] * inv, acc[8 * x + 7] * inv));
+            for (int rr = 0; rr < 4; ++rr) {
+                const int j = kTileM * a.t + r0 + rr;
+                if (j < pf.p_t) {
+                    const float inv = 1.0f / W[rr];
+                    uint2 pk;
+                    pk.x = pack_bf16(acc[rr].x * inv, acc[rr].y * inv);
+                    pk.y = pack_bf16(acc[rr].z * inv, acc[rr].w * inv);
+                    reinterpret_cast<uint2 *>(P.out + ((size_t)(pf.token_base + j) * P.hq + a.hq0 + e) *
+                                                          kHeadDim)[lane] = pk;
+                }
+            }
         }
     }
     if (tid == 0)
