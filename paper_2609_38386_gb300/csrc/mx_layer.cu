@@ -68,6 +68,7 @@ static_assert(sizeof(Misc) <= kSmemMiscBytes, "misc block too large");
 // Named barriers: 1 = every thread of the CTA between items, 2 = the 256
 // consumer threads (0 is __syncthreads, used only outside the item loops).
 constexpr uint32_t kBarItem = 1, kBarCons = 2;
+constexpr uint32_t kBarHead0 = 3;   // kBarHead0 + e: the 128 threads of head slot e's softmax
 __device__ __forceinline__ void cons_sync() { named_sync(kBarCons, kConsThreads); }
 
 // Instruction descriptors: S = Q K^T (both K-major) and O = P V (V MN-major).
@@ -1054,23 +1055,55 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
     tc_fence_after();
     const float inv = 1.0f / l_run;
     if (a.ns > 1) {
-        // one piece of a split tile: normalised partial O and its lse
+        // One piece of a split tile: normalised partial O and its lse.  O
+        // goes through shared memory (head 0 the K ring, head 1 the V ring:
+        // odone means every MMA of the item, so every load into the rings,
+        // has completed, and the next item's loads start only after the
+        // item boundary), so that each global write is a whole 512-byte row
+        // rather than one 16-byte piece of 32 rows.  A row's 16-byte chunk c
+        // sits at chunk c ^ (row & 31): writes by rows and reads along a row
+        // are both free of bank conflicts.
         const int part_slot = a.part_base + e * a.ns + a.s;
-        float *prow = P.pre_o + ((size_t)part_slot * kTileM + r) * kHeadDim;
+        const uint32_t stg = sbase + (e == 0 ? kSmemK : kSmemV);
 #pragma unroll
         for (int gq = 0; gq < 4; ++gq) {
             uint32_t o[32];
             tmem_ld32(tO + 32 * gq, o);
             tmem_wait_ld();
 #pragma unroll
-            for (int x = 0; x < 8; ++x)
-                reinterpret_cast<float4 *>(prow + 32 * gq)[x] =
-                    make_float4(__uint_as_float(o[4 * x]) * inv, __uint_as_float(o[4 * x + 1]) * inv,
-                                __uint_as_float(o[4 * x + 2]) * inv, __uint_as_float(o[4 * x + 3]) * inv);
+            for (int x = 0; x < 8; ++x) {
+                const uint32_t addr = stg + r * 512 + (((gq * 8 + x) ^ (r & 31)) << 4);
+                asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
+                             "f"(__uint_as_float(o[4 * x]) * inv), "f"(__uint_as_float(o[4 * x + 1]) * inv),
+                             "f"(__uint_as_float(o[4 * x + 2]) * inv), "f"(__uint_as_float(o[4 * x + 3]) * inv)
+                             : "memory");
+            }
         }
         float lg;
         asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(lg) : "f"(l_run));
         P.pre_lse[(size_t)part_slot * kTileM + r] = m_run + lg;
+        if (e == 0)   // the head's 128 rows are staged (barrier ids fixed at compile time)
+            named_sync(kBarHead0, kTileM);
+        else
+            named_sync(kBarHead0 + 1, kTileM);
+        // warp q4 of the head writes rows [32 q4, 32 q4 + 32), four at a time
+        const int lane = r & 31;
+        float *pbase = P.pre_o + (size_t)part_slot * kTileM * kHeadDim;
+#pragma unroll 1
+        for (int rr = 0; rr < 32; rr += 4) {
+            float4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int row = q4 * 32 + rr + u;
+                const uint32_t addr = stg + row * 512 + ((lane ^ (row & 31)) << 4);
+                asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                             : "=f"(v[u].x), "=f"(v[u].y), "=f"(v[u].z), "=f"(v[u].w)
+                             : "r"(addr));
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                reinterpret_cast<float4 *>(pbase + (size_t)(q4 * 32 + rr + u) * kHeadDim)[lane] = v[u];
+        }
         __threadfence();
         return;
     }
