@@ -1108,6 +1108,57 @@ __device__ void prefill_softmax(const LayerParams &P, uint8_t *smem, Misc *misc,
         return;
     }
     uint16_t *orow = P.out + ((size_t)(tb + j) * P.hq + hq) * kHeadDim;
+    if (!(a.t == 0 && cs < kShortRowKeys)) {
+        // No short rows to recompute from the tiles, so the head's Q tile
+        // (read by its last MMA, complete at odone) stages the bf16 rows and
+        // the warps write whole 256-byte rows, two per instruction.  A row's
+        // 16-byte chunk c sits at chunk c ^ (row & 15): conflict-free both
+        // ways.
+        const uint32_t stg = sbase + kSmemQ + e * kTileBytes;
+#pragma unroll
+        for (int gq = 0; gq < 4; ++gq) {
+            uint32_t o[32];
+            tmem_ld32(tO + 32 * gq, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                const uint32_t addr = stg + r * 256 + (((gq * 4 + x) ^ (r & 15)) << 4);
+                asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
+                             "r"(pack_bf16(__uint_as_float(o[8 * x + 0]) * inv, __uint_as_float(o[8 * x + 1]) * inv)),
+                             "r"(pack_bf16(__uint_as_float(o[8 * x + 2]) * inv, __uint_as_float(o[8 * x + 3]) * inv)),
+                             "r"(pack_bf16(__uint_as_float(o[8 * x + 4]) * inv, __uint_as_float(o[8 * x + 5]) * inv)),
+                             "r"(pack_bf16(__uint_as_float(o[8 * x + 6]) * inv, __uint_as_float(o[8 * x + 7]) * inv))
+                             : "memory");
+            }
+        }
+        if (e == 0)
+            named_sync(kBarHead0, kTileM);
+        else
+            named_sync(kBarHead0 + 1, kTileM);
+        // warp q4 of the head writes rows [32 q4, 32 q4 + 32), two per
+        // instruction (lanes 0-15 and 16-31), eight rows per round
+        const int lane = r & 31, half = lane >> 4, c = lane & 15;
+#pragma unroll 1
+        for (int rr = 0; rr < 32; rr += 8) {
+            uint4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int row = q4 * 32 + rr + 2 * u + half;
+                const uint32_t addr = stg + row * 256 + ((c ^ (row & 15)) << 4);
+                asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                             : "=r"(v[u].x), "=r"(v[u].y), "=r"(v[u].z), "=r"(v[u].w)
+                             : "r"(addr));
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int row = q4 * 32 + rr + 2 * u + half;
+                const int jr = kTileM * a.t + row;
+                if (jr < p)
+                    reinterpret_cast<uint4 *>(P.out + ((size_t)(tb + jr) * P.hq + hq) * kHeadDim)[c] = v[u];
+            }
+        }
+        return;
+    }
 #pragma unroll
     for (int gq = 0; gq < 4; ++gq) {
         uint32_t o[32];
