@@ -344,6 +344,18 @@ struct WorkList {
     int n_items = 0, n_prefill = 0, n_prefills = 0, split_keys = 0, piece_tiles = 0, v_stages = 2, dec_ctas = 0;
 };
 
+// Key pieces of query tile t of a chunk at chunk_start with nT key tiles.
+// A prompt's first tile at chunk_start < kShortRowKeys stays whole: its rows
+// of at most 16 keys are recomputed exactly in fp32 from the key tiles the
+// item holds (with so few keys, P rounded to bf16 would show in the output),
+// and a piece would hold only some of them.
+int tile_pieces(int chunk_start, int t, int nT, int piece)
+{
+    if (t == 0 && chunk_start < kShortRowKeys)
+        return 1;
+    return (nT + piece - 1) / piece;
+}
+
 // a1: the per-iteration work list, on the host, into dec[n_decodes] and
 // items[].  Prefill tiles first, heaviest (latest rows, most keys) first;
 // then decode splits, longest first.
@@ -417,7 +429,7 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
         for (const PrefillInfo &x : pfs) {
             const int nA = (x.chunk_start + kTileN - 1) / kTileN;
             for (int t = 0; t < (x.p_t + kTileM - 1) / kTileM; ++t) {
-                const int ns = (nA + t + 1 + pc - 1) / pc;
+                const int ns = tile_pieces(x.chunk_start, t, nA + t + 1, pc);
                 if (ns > 1)
                     parts += (int64_t)ns * hq;   // one partial per piece and head
             }
@@ -435,7 +447,7 @@ int build_work_list(const mx_geom &g, const mx_iter_desc *d, const PlanKnobs &k,
         const int nA = (pfs[f].chunk_start + kTileN - 1) / kTileN;
         for (int t = (pfs[f].p_t + kTileM - 1) / kTileM - 1; t >= 0; --t) {
             const int nT = nA + t + 1;
-            const int ns = (nT + piece - 1) / piece;
+            const int ns = tile_pieces(pfs[f].chunk_start, t, nT, piece);
             for (int gq = 0; gq < n_grp; ++gq) {
                 const int base = ns > 1 ? pre_part : 0;
                 if (ns > 1)

@@ -329,3 +329,19 @@ def test_a_sequence_takes_part_once():
     plan_work(decode_seq_ids=[0, 3], decode_ctx_lens=[5, 6], prefills=[(1, 0, 10), (2, 0, 10)], **base)
     plan_work(decode_seq_ids=[0, 3], decode_ctx_lens=[5, 6], prefill_seq_id=3, p_t=0, **base)
 
+
+
+@pytest.mark.parametrize("cs", [0, 5, 15, 16, 200])
+def test_first_tile_of_a_prompt_stays_whole(cs):
+    """A prompt's first query tile at chunk_start < 16 is never cut into key
+    pieces, even with the smallest piece option: its rows of at most 16 keys
+    are recomputed exactly from the key tiles the item holds.  Other tiles
+    are cut as the option says."""
+    pl = _plan(16, [], cs, 300, piece_tiles=1)
+    pre, _ = _decode_items(pl["items"])
+    n_a = -(-cs // TILE)
+    for d in pre:
+        n_t = n_a + d["t"] + 1
+        want = 1 if (d["t"] == 0 and cs < 16) else n_t
+        assert d["ns"] == want, (cs, d)
+    _check(pl, 16, [], cs, 300)
