@@ -18,7 +18,7 @@
  *    attention, and §4.3/§5.1 require outputs to agree exactly with and
  *    without chunking.
  *
- * Readings where the paper is silent (listed in the design notes as well):
+ * Readings where the paper is silent:
  *  - softmax scale 1/sqrt(head_dim);
  *  - GQA: query head h reads KV head h / (Hq/Hkv);
  *  - a decode with ctx cached tokens attends ctx + 1 keys (its own new key);
