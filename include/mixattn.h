@@ -213,7 +213,10 @@ int mx_error_detail(mx_ctx *ctx, char *buf, int32_t len);
  * 0 = automatic).  MX_OPT_GRID: persistent grid size (0 = number of SMs).
  * MX_OPT_PREFILL_PIECE_TILES: at most this many 128-key tiles per prefill
  * work item; longer causal tiles are split into pieces merged by
- * log-sum-exp (0 = automatic, 65535 = never split). */
+ * log-sum-exp (0 = automatic, 65535 = never split).  A prompt's first query
+ * tile at chunk_start < 16 is never split (its rows of at most 16 keys are
+ * recomputed exactly from the tiles the item holds); the size doubles while
+ * the pieces' partials would not fit the context's workspace. */
 #define MX_OPT_SPLIT_KEYS 1
 #define MX_OPT_GRID 2
 #define MX_OPT_PREFILL_PIECE_TILES 3
